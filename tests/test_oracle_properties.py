@@ -1,0 +1,169 @@
+"""Invariants that pin the oracle's passes (no printed logits exist to compare with).
+
+- Exact verification (Section 4.1, Appendix A.1): speculative output equals greedy
+  decoding by the adapter-off verifier, for any drafter.
+- B = 0 and D = 1 reduces PEFT-BD to greedy decoding with one accepted draft per round.
+- The draft's pending-token row sees only the cache and itself: with B = 0 its logits
+  equal the verify row's logits bit for bit.
+- The adapter-off path never reads A or B.
+- The mask rows attend to each other (bidirectional block), the pending row does not.
+- After any number of rounds, the committed KV equals a fresh prefill of the same tokens.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from oracle import MASK_BLOCK_DRAFT, MASK_CAUSAL
+
+
+@pytest.fixture(scope="module")
+def greedy64(tiny):
+    return oracle.greedy_generate(tiny["model"], tiny["prompt"], 64)
+
+
+@pytest.mark.parametrize("D", [1, 2, 4, 16])
+def test_spec_equals_greedy(tiny, greedy64, D):
+    out, rounds = oracle.spec_generate(tiny["model"], tiny["prompt"], 64, D)
+    assert out == greedy64
+
+
+def test_spec_equals_greedy_adversarial_drafters(tiny, greedy64):
+    m, prompt, V = tiny["model"], tiny["prompt"], tiny["shape"].vocab
+    D = 4
+    cont = greedy64 + [0] * (D + 2)
+
+    # all-correct: the drafter proposes the greedy continuation, so every round accepts
+    # n == D and emits D+1 tokens; round ri therefore starts at output position 1 + ri*(D+1)
+    def all_correct(ri, drafts):
+        pos = 1 + ri * (D + 1)
+        return cont[pos:pos + D]
+
+    out, rounds = oracle.spec_generate(m, prompt, 64, D, draft_override=all_correct)
+    pos = 1
+    for r in rounds:
+        assert r["draft"] == cont[pos:pos + D]
+        if pos + D <= len(greedy64):  # past the budget the drafter pads with zeros
+            assert r["n"] == D
+        pos += r["n"] + 1
+    assert out == greedy64
+
+    # all-wrong: every draft differs from the verifier (n == 0), one token per round
+    out, rounds = oracle.spec_generate(m, prompt, 64, D,
+                                       draft_override=lambda ri, d: [(t + 1) % V for t in d])
+    assert all(r["n"] == 0 for r in rounds)
+    assert out == greedy64
+
+    # random drafts: still exact
+    rng = np.random.default_rng(7)
+    out, rounds = oracle.spec_generate(m, prompt, 64, D,
+                                       draft_override=lambda ri, d: list(rng.integers(0, V, size=D)))
+    assert out == greedy64
+
+
+def test_zero_B_d1_is_greedy_with_one_accepted(tiny_zeroB):
+    m, prompt = tiny_zeroB["model"], tiny_zeroB["prompt"]
+    g = oracle.greedy_generate(m, prompt, 40)
+    out, rounds = oracle.spec_generate(m, prompt, 40, 1)
+    assert out == g
+    assert all(r["n"] == 1 for r in rounds[:-1])
+
+
+def test_zero_B_anchor_row_equals_verify_row(tiny_zeroB):
+    m, prompt = tiny_zeroB["model"], tiny_zeroB["prompt"]
+    P, D = len(prompt), 16
+    cache, p, _ = m.prefill(prompt, P + 64)
+    _, dl, _ = m.forward(cache, P, [p] + [-1] * D, True, MASK_BLOCK_DRAFT, 0, D, want_logits=True)
+    _, vl, _ = m.forward(cache, P, [p] + [3] * D, False, MASK_CAUSAL, 0, D + 1, want_logits=True)
+    assert np.array_equal(dl[0].view(np.uint32), vl[0].view(np.uint32))
+    # and with B = 0 every spec round accepts at least the first draft
+    out, rounds = oracle.spec_generate(m, prompt, 48, D)
+    assert all(r["n"] >= 1 for r in rounds)
+
+
+def test_adapter_off_ignores_A_and_B(tiny):
+    from paper_2607_12422_gb300 import synth
+    S = tiny["shape"]
+    nan_ad = {k: np.full_like(v, 0x7FC0) for k, v in tiny["adapter"].items()}
+    nan_ad["mask_embed"] = tiny["adapter"]["mask_embed"]
+    m2 = oracle.OracleModel(S, tiny["base"], nan_ad)
+    prompt = tiny["prompt"][:40]
+    c1 = tiny["model"].new_cache(64)
+    c2 = m2.new_cache(64)
+    _, l1, _ = tiny["model"].forward(c1, 0, prompt, False, MASK_CAUSAL, 0, 40, want_logits=True)
+    _, l2, _ = m2.forward(c2, 0, prompt, False, MASK_CAUSAL, 0, 40, want_logits=True)
+    assert np.array_equal(l1.view(np.uint32), l2.view(np.uint32))
+    # adapter on with NaN factors does poison the result (the flag really switches the delta)
+    _, l3, _ = m2.forward(c2, 0, prompt, True, MASK_CAUSAL, 0, 40, want_logits=True)
+    assert np.isnan(l3).all()
+
+
+def test_block_mask_structure(tiny):
+    m, prompt = tiny["model"], tiny["prompt"]
+    P, D = len(prompt), 8
+    cache, p, _ = m.prefill(prompt, P + 64)
+    base_rows = [p] + [-1] * D
+    _, l0, _ = m.forward(cache, P, base_rows, True, MASK_BLOCK_DRAFT, 0, D + 1, want_logits=True)
+    # change only the last row's input: every other mask row must change, the pending row must not
+    alt = list(base_rows)
+    alt[-1] = 17
+    _, l1, _ = m.forward(cache, P, alt, True, MASK_BLOCK_DRAFT, 0, D + 1, want_logits=True)
+    assert np.array_equal(l0[0], l1[0])
+    for j in range(1, D):
+        assert not np.array_equal(l0[j], l1[j]), j
+    # under the causal mask the same change leaves rows 0..D-1 untouched
+    _, c0, _ = m.forward(cache, P, base_rows, True, MASK_CAUSAL, 0, D + 1, want_logits=True)
+    _, c1, _ = m.forward(cache, P, alt, True, MASK_CAUSAL, 0, D + 1, want_logits=True)
+    assert np.array_equal(c0[:D], c1[:D])
+
+
+def test_mask_embedding_reaches_mask_rows_only(tiny):
+    S = tiny["shape"]
+    ad2 = dict(tiny["adapter"])
+    me = ad2["mask_embed"].copy()
+    me[:16] ^= 0x0100  # flip a mantissa bit of a few elements
+    ad2["mask_embed"] = me
+    m2 = oracle.OracleModel(S, tiny["base"], ad2)
+    m, prompt = tiny["model"], tiny["prompt"]
+    P, D = len(prompt), 8
+    cache, p, _ = m.prefill(prompt, P + 64)
+    cache2, p2, _ = m2.prefill(prompt, P + 64)
+    assert p == p2
+    _, a, _ = m.forward(cache, P, [p] + [-1] * D, True, MASK_BLOCK_DRAFT, 0, D + 1, want_logits=True)
+    _, b, _ = m2.forward(cache2, P, [p] + [-1] * D, True, MASK_BLOCK_DRAFT, 0, D + 1, want_logits=True)
+    assert np.array_equal(a[0], b[0])
+    assert all(not np.array_equal(a[j], b[j]) for j in range(1, D + 1))
+
+
+def test_kv_after_rounds_equals_fresh_prefill(tiny):
+    m, prompt, S = tiny["model"], tiny["prompt"], tiny["shape"]
+    D = 4
+    rng = np.random.default_rng(3)
+    forced = list(rng.integers(0, D + 1, size=64))
+    out, rounds, (cache, L) = oracle.spec_generate(m, prompt, 30, D, forced_n=forced, return_state=True)
+    seq = list(prompt) + out[:-1]
+    # the committed length covers the prompt and every emitted token but the pending one
+    assert L == len(seq) or L > len(seq)  # the last round may be truncated by the budget
+    n_chk = len(seq)
+    fresh = m.new_cache(len(seq) + 8)
+    m.forward(fresh, 0, seq, False, MASK_CAUSAL, len(seq) - 1, 1)
+    for layer in range(S.n_layers):
+        for which in ("k", "v"):
+            a = cache.read(layer, which, n_chk)
+            b = fresh.read(layer, which, n_chk)
+            assert np.array_equal(a.view(np.uint32), b.view(np.uint32)), (layer, which)
+
+
+def test_forced_n_spec_is_kv_consistent_not_greedy(tiny):
+    """Forced acceptance commits d_1..d_n, v_n; the next rounds must continue from that state."""
+    m, prompt = tiny["model"], tiny["prompt"][:20]
+    D = 4
+    forced = [D, 0, 2, D, 1, 3] * 10
+    out, rounds = oracle.spec_generate(m, prompt, 40, D, forced_n=forced)
+    assert [r["n"] for r in rounds] == forced[:len(rounds)]
+    # replaying the committed tokens with plain causal passes gives each round's verify tokens
+    seq = list(prompt) + [out[0]]
+    for r in rounds[:4]:
+        cache = m.new_cache(len(seq) + D + 2)
+        am, _, _ = m.forward(cache, 0, seq + r["draft"], False, MASK_CAUSAL, len(seq) - 1, D + 1)
+        assert list(am) == r["verify"]
+        seq = seq + r["emitted"]
