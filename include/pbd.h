@@ -156,6 +156,26 @@ pbd_status pbd_read_kv(pbd_ctx *ctx, int32_t layer, int32_t seq, int32_t n, void
 /* Waits for the stream and reports a latched device error. */
 pbd_status pbd_sync(pbd_ctx *ctx);
 
+/* Timing of the decode loop (the profile of Appendix A.5 measures draft and verify forward
+ * latency separately).  On a prefilled context, replays `warmup` untimed and then `steps` timed
+ * rounds, each as CUDA graphs on the context's stream: mode 0 = draft pass, verify pass,
+ * accept/commit; mode 1 = one plain greedy step (verify-style pass of one row, commit).
+ * CUDA events bracket each phase of every timed round.  h_ms[0..3] receive the summed ms of
+ * the draft passes, the verify (or AR) passes, the commits, and the whole timed region;
+ * h_launches receives the kernels launched per round.  d_forced_n_seq_opt as in pbd_generate
+ * (indexed by round from the start of the call).  Synchronous on return. */
+pbd_status pbd_bench_rounds(pbd_ctx *ctx, int32_t mode, int32_t warmup, int32_t steps,
+                            const int32_t *d_forced_n_seq_opt, double *h_ms, int32_t *h_launches);
+
+/* Times the tensor-core linear kernel alone: for `iters` sweeps over all layers, launches the
+ * projection `which` (0 q|k|v, 1 o, 2 gate|up, 3 down; 4 the lm_head, once per sweep) with `rows`
+ * token rows and the adapter rows on or off, back to back on the context's stream.  Successive
+ * launches read different layers' weights (larger than L2 in total).  *h_ms_per_launch receives
+ * the mean launch duration from CUDA events; *h_weight_bytes the weight bytes one launch reads.
+ * Buffers hold whatever the last pass left; only the timing is meaningful. */
+pbd_status pbd_time_linear(pbd_ctx *ctx, int32_t which, int32_t rows, int32_t adapter, int32_t iters,
+                           double *h_ms_per_launch, double *h_weight_bytes);
+
 const char *pbd_last_error(const pbd_ctx *ctx);
 
 /* Build/version tag of the library ("pbd sm_103a <date>"). */

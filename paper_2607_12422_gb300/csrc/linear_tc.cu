@@ -170,8 +170,7 @@ __global__ void __launch_bounds__(LIN_THREADS, 1)
     }
     if constexpr (EPI == EPI_ARGMAX) {
         __syncthreads();
-        if (have && threadIdx.x < BN && tok0 + (int)threadIdx.x < M) {
-            const int c = threadIdx.x;
+        for (int c = threadIdx.x; have && c < BN && tok0 + c < M; c += LIN_THREADS) {
             float bv = red_val[c];
             int bi = red_idx[c];
             for (int w = 1; w < 4; ++w) {

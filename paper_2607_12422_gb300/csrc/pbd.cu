@@ -95,6 +95,23 @@ struct pbd_ctx {
     int batch = 0, max_new = 0;
     Phase phase = PH_NONE;
     std::string err;
+    // graphs of pbd_bench_rounds, reused while batch size and forced table are unchanged
+    cudaGraphExec_t bench_gx[2][3] = {{nullptr, nullptr, nullptr}, {nullptr, nullptr, nullptr}};
+    const int32_t *bench_forced[2] = {nullptr, nullptr};
+    int bench_batch[2] = {0, 0};
+    size_t bench_nodes[2] = {0, 0};
+    void drop_bench_graphs(int mode) {
+        for (auto &g : bench_gx[mode])
+            if (g) {
+                cudaGraphExecDestroy(g);
+                g = nullptr;
+            }
+        bench_batch[mode] = 0;
+    }
+    ~pbd_ctx() {
+        drop_bench_graphs(0);
+        drop_bench_graphs(1);
+    }
 };
 
 namespace {
@@ -724,6 +741,153 @@ pbd_status pbd_read_kv(pbd_ctx *c, int32_t layer, int32_t seq, int32_t n, void *
 
 pbd_status pbd_sync(pbd_ctx *c) {
     if (!c) return fail(c, PBD_ERR_INVALID_ARG, "null context");
+    return check_device(c);
+}
+
+pbd_status pbd_bench_rounds(pbd_ctx *c, int32_t mode, int32_t warmup, int32_t steps, const int32_t *d_forced_n_seq_opt,
+                            double *h_ms, int32_t *h_launches) {
+    if (!c || !h_ms) return fail(c, PBD_ERR_INVALID_ARG, "null argument");
+    if (mode != 0 && mode != 1) return fail(c, PBD_ERR_INVALID_ARG, "mode must be 0 or 1");
+    if (steps < 1 || warmup < 0) return fail(c, PBD_ERR_INVALID_ARG, "steps must be >= 1");
+    if (c->phase != PH_READY) return fail(c, PBD_ERR_STATE, "bench needs a prefilled or committed state");
+    if (c->st == nullptr || c->st == cudaStreamLegacy)
+        return fail(c, PBD_ERR_INVALID_ARG, "bench needs a non-default stream (graph capture)");
+    CK(cudaMemsetAsync(c->s.round, 0, sizeof(int), c->st));
+    const int nph = 3;
+    cudaGraphExec_t *gx = c->bench_gx[mode];
+    const bool cached = c->bench_batch[mode] == c->batch && c->bench_forced[mode] == d_forced_n_seq_opt &&
+                        gx[mode == 0 ? 0 : 1] != nullptr;
+    if (!cached) c->drop_bench_graphs(mode);
+    size_t nodes = cached ? c->bench_nodes[mode] : 0;
+    pbd_status s = PBD_OK;
+    for (int ph = 0; ph < nph && s == PBD_OK && !cached; ++ph) {
+        if (mode == 1 && ph == 0) continue;  // no draft phase in plain decoding
+        cudaGraph_t g = nullptr;
+        CK(cudaStreamBeginCapture(c->st, cudaStreamCaptureModeThreadLocal));
+        if (mode == 0) {
+            if (ph == 0) s = enqueue_draft(c, nullptr);
+            if (ph == 1) s = enqueue_verify(c, c->draft_ids, nullptr);
+            if (ph == 2) s = enqueue_accept(c, d_forced_n_seq_opt, nullptr);
+        } else {
+            const PassDesc pd = block_pass(c, PK_DECODE);
+            if (ph == 1) {
+                cudaError_t e = launch_build_ids(pd, 2, c->s.pending, nullptr, 0, c->ids, c->st);
+                s = e == cudaSuccess ? run_pass(c, pd, c->verify_ids, nullptr)
+                                     : fail(c, PBD_ERR_CUDA, "build ids: %s", cudaGetErrorString(e));
+            }
+            if (ph == 2) {
+                cudaError_t e = launch_accept_commit(c->s, c->batch, 0, c->draft_ids, c->verify_ids, nullptr,
+                                                     c->batch, c->max_new, c->out_cap, nullptr, c->st);
+                if (e != cudaSuccess) s = fail(c, PBD_ERR_CUDA, "accept: %s", cudaGetErrorString(e));
+            }
+        }
+        cudaError_t e = cudaStreamEndCapture(c->st, &g);
+        if (s == PBD_OK && e != cudaSuccess) s = fail(c, PBD_ERR_CUDA, "capture: %s", cudaGetErrorString(e));
+        if (s == PBD_OK) {
+            size_t n = 0;
+            cudaGraphGetNodes(g, nullptr, &n);
+            nodes += n;
+            e = cudaGraphInstantiate(&gx[ph], g, 0);
+            if (e != cudaSuccess) s = fail(c, PBD_ERR_CUDA, "instantiate: %s", cudaGetErrorString(e));
+        }
+        if (g) cudaGraphDestroy(g);
+    }
+    if (s != PBD_OK) {
+        c->drop_bench_graphs(mode);
+        return s;
+    }
+    if (!cached) {
+        c->bench_batch[mode] = c->batch;
+        c->bench_forced[mode] = d_forced_n_seq_opt;
+        c->bench_nodes[mode] = nodes;
+    }
+    std::vector<cudaEvent_t> ev;
+    if (s == PBD_OK) {
+        ev.resize((size_t)steps * 4, nullptr);
+        for (auto &x : ev)
+            if (cudaEventCreate(&x) != cudaSuccess) s = fail(c, PBD_ERR_CUDA, "event create");
+    }
+    for (int i = 0; s == PBD_OK && i < warmup + steps; ++i) {
+        const bool timed = i >= warmup;
+        cudaEvent_t *e4 = timed ? &ev[(size_t)(i - warmup) * 4] : nullptr;
+        for (int ph = 0; ph < nph; ++ph) {
+            if (timed) cudaEventRecord(e4[ph], c->st);
+            if (gx[ph] && cudaGraphLaunch(gx[ph], c->st) != cudaSuccess) {
+                s = fail(c, PBD_ERR_CUDA, "graph launch");
+                break;
+            }
+        }
+        if (timed) cudaEventRecord(e4[3], c->st);
+    }
+    if (s == PBD_OK && cudaStreamSynchronize(c->st) != cudaSuccess) s = fail(c, PBD_ERR_CUDA, "bench sync");
+    if (s == PBD_OK) {
+        double acc[3] = {0, 0, 0};
+        for (int i = 0; i < steps; ++i)
+            for (int ph = 0; ph < 3; ++ph) {
+                float ms = 0.f;
+                cudaEventElapsedTime(&ms, ev[(size_t)i * 4 + ph], ev[(size_t)i * 4 + ph + 1]);
+                acc[ph] += ms;
+            }
+        float tot = 0.f;
+        cudaEventElapsedTime(&tot, ev[0], ev[(size_t)(steps - 1) * 4 + 3]);
+        h_ms[0] = acc[0];
+        h_ms[1] = acc[1];
+        h_ms[2] = acc[2];
+        h_ms[3] = tot;
+        if (h_launches) *h_launches = (int32_t)nodes;
+    }
+    for (auto &x : ev)
+        if (x) cudaEventDestroy(x);
+    if (s != PBD_OK) {
+        c->drop_bench_graphs(mode);
+        return s;
+    }
+    c->phase = PH_READY;
+    return check_device(c);
+}
+
+pbd_status pbd_time_linear(pbd_ctx *c, int32_t which, int32_t rows, int32_t adapter, int32_t iters,
+                           double *h_ms_per_launch, double *h_weight_bytes) {
+    if (!c || !h_ms_per_launch) return fail(c, PBD_ERR_INVALID_ARG, "null argument");
+    if (which < 0 || which > 4 || iters < 1) return fail(c, PBD_ERR_INVALID_ARG, "which in [0,4], iters >= 1");
+    const int max_rows = which == 4 ? c->ro_alloc : c->rows_alloc;
+    if (rows < 1 || rows > max_rows) return fail(c, PBD_ERR_CAPACITY, "rows outside [1, %d]", max_rows);
+    const int bn = pick_bn(rows), bi = bn_index(bn);
+    const int nl = c->cfg.n_layers;
+    const int per_sweep = which == 4 ? 1 : nl;
+    auto launch = [&](int l) -> cudaError_t {
+        switch (which) {
+            case 0: return launch_linear_partials(&c->maps[AB_X][bi], bn, c->w_qkv[l], adapter, rows,
+                                                  partials_for(c, c->w_qkv[l]), c->status, c->st);
+            case 1: return launch_linear_partials(&c->maps[AB_ATTN][bi], bn, c->w_o[l], adapter, rows,
+                                                  partials_for(c, c->w_o[l]), c->status, c->st);
+            case 2: return launch_linear_partials(&c->maps[AB_X][bi], bn, c->w_gu[l], adapter, rows,
+                                                  partials_for(c, c->w_gu[l]), c->status, c->st);
+            case 3: return launch_linear_partials(&c->maps[AB_ACT][bi], bn, c->w_down[l], adapter, rows,
+                                                  partials_for(c, c->w_down[l]), c->status, c->st);
+            default: return launch_lm_head(&c->maps[AB_XRO][bi], bn, c->w_lm, rows, c->tile_max, c->tile_arg,
+                                           nullptr, c->status, c->st);
+        }
+    };
+    for (int l = 0; l < per_sweep; ++l) CK(launch(l));  // warm-up sweep
+    cudaEvent_t e0, e1;
+    CK(cudaEventCreate(&e0));
+    CK(cudaEventCreate(&e1));
+    CK(cudaEventRecord(e0, c->st));
+    for (int it = 0; it < iters; ++it)
+        for (int l = 0; l < per_sweep; ++l) CK(launch(l));
+    CK(cudaEventRecord(e1, c->st));
+    CK(cudaEventSynchronize(e1));
+    float ms = 0.f;
+    cudaEventElapsedTime(&ms, e0, e1);
+    cudaEventDestroy(e0);
+    cudaEventDestroy(e1);
+    *h_ms_per_launch = (double)ms / ((double)iters * per_sweep);
+    if (h_weight_bytes) {
+        const TiledWeight &w = which == 0 ? c->w_qkv[0] : which == 1 ? c->w_o[0] : which == 2 ? c->w_gu[0]
+                               : which == 3 ? c->w_down[0] : c->w_lm;
+        *h_weight_bytes = 2.0 * (double)w.K * (w.n_main + (adapter && which < 4 ? w.lora_rows : 0));
+    }
     return check_device(c);
 }
 

@@ -90,6 +90,10 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     L.pbd_last_error.restype = C.c_char_p
     L.pbd_last_error.argtypes = [P]
     L.pbd_version.restype = C.c_char_p
+    L.pbd_bench_rounds.argtypes = [P, I32, I32, I32, P, P, P]
+    L.pbd_time_linear.argtypes = [P, I32, I32, I32, I32, P, P]
+    L.pbd_bench_rounds.restype = C.c_int
+    L.pbd_time_linear.restype = C.c_int
     L.pbd_op_linear_workspace_bytes.restype = C.c_size_t
     L.pbd_op_linear_workspace_bytes.argtypes = [I32, I32, I32, I32]
     L.pbd_op_linear.argtypes = [I32, I32, I32, I32, C.c_float, P, P, P, P, P, P, C.c_size_t, P]
@@ -328,3 +332,21 @@ class Engine:
 
     def pbd_sync(self):
         self._call(self.lib.pbd_sync)
+
+    def pbd_bench_rounds(self, mode: int, warmup: int, steps: int, forced_n_seq=None):
+        """Returns (ms_draft, ms_verify_or_ar, ms_commit, ms_total, launches_per_round) summed over the steps."""
+        ms = np.zeros(4, np.float64)
+        launches = np.zeros(1, np.int32)
+        fp = None
+        if forced_n_seq is not None:
+            forced_n_seq = self.torch.as_tensor(forced_n_seq, dtype=self.torch.int32).to(self.device).contiguous()
+            fp = forced_n_seq.data_ptr()
+        self._call(self.lib.pbd_bench_rounds, mode, warmup, steps, fp, ms.ctypes.data, launches.ctypes.data)
+        return float(ms[0]), float(ms[1]), float(ms[2]), float(ms[3]), int(launches[0])
+
+    def pbd_time_linear(self, which: int, rows: int, adapter: int, iters: int):
+        """(ms per launch, weight bytes per launch) of the tensor-core linear kernel timed alone."""
+        ms = np.zeros(1, np.float64)
+        wb = np.zeros(1, np.float64)
+        self._call(self.lib.pbd_time_linear, which, rows, adapter, iters, ms.ctypes.data, wb.ctypes.data)
+        return float(ms[0]), float(wb[0])

@@ -97,9 +97,12 @@ WORKLOADS = {
 def bf16_bits(x: np.ndarray) -> np.ndarray:
     """float32 -> bfloat16 bit patterns by IEEE round-to-nearest-even (data encoding only)."""
     u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
-    lsb = (u >> 16) & np.uint32(1)
-    r = ((u + np.uint32(0x7FFF) + lsb) >> 16).astype(np.uint16)
-    return r
+    lsb = u >> 16
+    lsb &= np.uint32(1)
+    w = u + np.uint32(0x7FFF)
+    w += lsb
+    w >>= 16
+    return w.astype(np.uint16)
 
 
 def bf16_to_f32(b: np.ndarray) -> np.ndarray:
@@ -110,10 +113,13 @@ def _normal_bf16(rng: np.random.Generator, shape, std: float = INIT_STD) -> np.n
     out = np.empty(shape, dtype=np.uint16)
     flat = out.reshape(-1)
     n = flat.size
-    chunk = 1 << 24
+    chunk = 1 << 22
+    buf = np.empty(min(n, chunk), dtype=np.float32)
     for s in range(0, n, chunk):
         e = min(n, s + chunk)
-        v = rng.standard_normal(e - s, dtype=np.float32) * np.float32(std)
+        v = buf[: e - s]
+        rng.standard_normal(out=v, dtype=np.float32)
+        v *= np.float32(std)
         flat[s:e] = bf16_bits(v)
     return out
 

@@ -73,7 +73,8 @@ def test_linear_matches_oracle(torch_dev, M, K, N, r):
     assert (got == ref).mean() > 0.95
 
 
-@pytest.mark.parametrize("M,H,V", [(1, 1024, 4096), (17, 1024, 151936 // 8), (16, 256, 4096), (136, 1024, 2048)])
+@pytest.mark.parametrize("M,H,V", [(1, 1024, 4096), (17, 1024, 18944), (16, 256, 4096), (136, 1024, 2048),
+                                   (200, 256, 1024)])
 def test_lm_head_argmax_matches_oracle(torch_dev, M, H, V):
     from paper_2607_12422_gb300 import pbd
     torch = torch_dev
