@@ -255,6 +255,13 @@ def main(args):
         return acc, tokens, launches, l_sum / steps
 
     hbm, peak_kind = peaks()
+    if args.profile_rounds:
+        # profiler configuration: prefill, then warm-up and timed rounds only (no other legs)
+        acc, tokens, launches, L_mean = timed_rounds(0, args.steps, args.warmup)
+        print(json.dumps({"profile_rounds": args.steps, "ms_per_step": acc[3] / args.steps,
+                          "launches_per_round": launches // args.steps}))
+        eng.close()
+        return 0
     # ---- main measurement: speculative rounds
     if dist:
         dist.barrier()
@@ -359,6 +366,8 @@ if __name__ == "__main__":
     ap.add_argument("--warmup", type=int, default=8)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile-rounds", action="store_true",
+                    help="only prefill + warm-up + timed rounds (the configuration profiled under ncu)")
     a = ap.parse_args()
     if a.warmup < 3:
         a.warmup = 3

@@ -60,13 +60,13 @@ class _Weights(C.Structure):
                 ("lora_b", _U16P * 7), ("mask_embed", _U16P)]
 
 
-_lib = None
+_libs = {}
 
 
-def lib():
-    global _lib
-    if _lib is None:
-        L = C.CDLL(build())
+def lib(variant: str = "f32"):
+    """The oracle library: 'f32' (reference) or 'f64acc' (fp64 accumulators, drift measurement only)."""
+    if variant not in _libs:
+        L = C.CDLL(build(variant=variant))
         F = C.POINTER(C.c_float)
         I32 = C.POINTER(C.c_int32)
         L.orc_cache_new.restype = C.c_void_p
@@ -88,8 +88,8 @@ def lib():
         L.orc_round_bf16.argtypes = [C.c_float]
         L.orc_round_bf16.restype = C.c_float
         L.orc_num_threads.restype = C.c_int32
-        _lib = L
-    return _lib
+        _libs[variant] = L
+    return _libs[variant]
 
 
 def _fp(a: np.ndarray):
@@ -145,8 +145,9 @@ class OracleCache:
 class OracleModel:
     """Holds the config and the bf16 weight arrays (uint16 bit patterns) for the C library."""
 
-    def __init__(self, shape, base: Dict[str, np.ndarray], adapter: Dict[str, np.ndarray]):
+    def __init__(self, shape, base: Dict[str, np.ndarray], adapter: Dict[str, np.ndarray], acc: str = "f32"):
         self.shape = shape
+        self.acc = acc
         self.cfg = make_config(shape)
         nl, r = shape.n_layers, shape.lora_rank
         keep = {}
@@ -192,7 +193,7 @@ class OracleModel:
         am = np.empty(n_read, dtype=np.int32)
         logits = np.empty((n_read, self.shape.vocab), dtype=np.float32) if want_logits else None
         hidden = np.empty((n_read, self.shape.hidden), dtype=np.float32) if want_hidden else None
-        rc = lib().orc_forward(C.byref(self.cfg), C.byref(self.weights), cache.ptr, L, n, _i32(toks),
+        rc = lib(self.acc).orc_forward(C.byref(self.cfg), C.byref(self.weights), cache.ptr, L, n, _i32(toks),
                                int(adapter_on), mask_mode, read_first, n_read,
                                _fp(logits) if logits is not None else None, _i32(am),
                                _fp(hidden) if hidden is not None else None)

@@ -110,15 +110,24 @@ static inline float round_bf16(float f) {
     return f;
 }
 
-/* Fixed-order fp32 sums: term k accumulates into partial k % 16, then a pairwise tree. */
-static inline float combine16(float s[16]) {
+/* Accumulator of every dot product: fp32 (the reference build).  Built with -DORC_ACC_DOUBLE
+ * the same sums run in fp64; the tests use that second build only to measure how far two
+ * valid summation orders of the bf16 model drift apart (the floor of any logit tolerance). */
+#ifdef ORC_ACC_DOUBLE
+typedef double acc_t;
+#else
+typedef float acc_t;
+#endif
+
+/* Fixed-order sums: term k accumulates into partial k % 16, then a pairwise tree. */
+static inline float combine16(acc_t s[16]) {
     for (int w = 8; w >= 1; w >>= 1)
         for (int j = 0; j < w; j++) s[j] = s[j] + s[j + w];
-    return s[0];
+    return (float)s[0];
 }
 
 static float dot_fw(const float *x, const uint16_t *w, int n) {
-    float s[16] = {0};
+    acc_t s[16] = {0};
     int k = 0;
     for (; k + 16 <= n; k += 16)
         for (int j = 0; j < 16; j++) s[j] = s[j] + x[k + j] * bf16_to_f32(w[k + j]);
@@ -127,7 +136,7 @@ static float dot_fw(const float *x, const uint16_t *w, int n) {
 }
 
 static float dot_ff(const float *x, const float *y, int n) {
-    float s[16] = {0};
+    acc_t s[16] = {0};
     int k = 0;
     for (; k + 16 <= n; k += 16)
         for (int j = 0; j < 16; j++) s[j] = s[j] + x[k + j] * y[k + j];
