@@ -110,7 +110,7 @@ class ClockSampler:
 
 def traffic_for(kernel_src):
     """DRAM bytes per launch from the committed ncu summary, if the kernel source is unchanged since."""
-    path = os.path.join(ROOT, "profiles", "linear_tc_gate_up_m17_traffic.json")
+    path = os.path.join(ROOT, "profiles", "k_pass_verify_qwen3_0.6b_traffic.json")
     try:
         with open(path) as f:
             rec = json.load(f)
@@ -297,11 +297,12 @@ def main(args):
     floor_v = b_verify / (hbm * 1e9) * 1e6
     floor_d = b_draft / (hbm * 1e9) * 1e6
 
-    # ---- dominant kernel: the tensor-core linear (gate|up, 17 rows, adapter off), timed alone over 28 layers
-    ms_lin, wbytes = eng.pbd_time_linear(2, D + 1, 0, 8)
-    lin_bytes = wbytes + 2 * (D + 1) * S.hidden + 2 * (D + 1) * 2 * S.intermediate
-    achieved = lin_bytes / (ms_lin * 1e-3) / 1e9
-    traffic = traffic_for(os.path.join(ROOT, "paper_2607_12422_gb300", "csrc", "linear_tc.cu"))
+    # ---- dominant kernel: the persistent pass kernel (all 28 layers of a verify pass), timed alone
+    eng.pbd_prefill([prompt], max_new=G)
+    ms_k, k_bytes = eng.pbd_time_pass(1, 16)
+    ms_kd, kd_bytes = eng.pbd_time_pass(0, 16)
+    achieved = k_bytes / (ms_k * 1e-3) / 1e9
+    traffic = traffic_for(os.path.join(ROOT, "paper_2607_12422_gb300", "csrc", "pass_kernel.cu"))
 
     # ---- end to end through the public call with host buffers
     # (host prompt ids in, host token ids out; the binding copies the prompt to the device)
@@ -340,10 +341,12 @@ def main(args):
                        "mean_tokens_per_round": mean_A, "draft_over_verify": draft_us / verify_us},
             "ar": {"us_per_step": ar_us, "pass_us": ar_pass_us, "tokens_per_s": tok_ar / (acc_ar[3] / 1e3),
                    "break_even_accept": (draft_us + verify_us) / ar_us},
-            "roofline": {"bound": "hbm", "kernel": "k_linear_tc<32,partial> gate|up 6144x1024, 17 rows",
+            "roofline": {"bound": "hbm", "kernel": "k_pass (persistent; 28 layers of one verify pass, 17 rows)",
                          "achieved": achieved, "peak": hbm, "peak_kind": peak_kind + " hbm_gbs (burst)",
                          "unit": "GB/s", "frac": achieved / hbm, "traffic": traffic,
-                         "algorithmic_bytes": lin_bytes, "us_per_launch": ms_lin * 1e3},
+                         "algorithmic_bytes": k_bytes, "us_per_launch": ms_k * 1e3,
+                         "draft_kernel": {"us_per_launch": ms_kd * 1e3, "algorithmic_bytes": kd_bytes,
+                                          "frac": kd_bytes / (ms_kd * 1e-3) / 1e9 / hbm}},
             "cpu_baseline": cpu,
             "e2e": {"value": e2e, "unit": "tokens/s", "h2d_bytes_per_step": 4 * P, "d2h_bytes_per_step": 4 * G,
                     "step": "one pbd_generate call (prefill + rounds) per generation"},

@@ -167,14 +167,15 @@ pbd_status pbd_sync(pbd_ctx *ctx);
 pbd_status pbd_bench_rounds(pbd_ctx *ctx, int32_t mode, int32_t warmup, int32_t steps,
                             const int32_t *d_forced_n_seq_opt, double *h_ms, int32_t *h_launches);
 
-/* Times the tensor-core linear kernel alone: for `iters` sweeps over all layers, launches the
- * projection `which` (0 q|k|v, 1 o, 2 gate|up, 3 down; 4 the lm_head, once per sweep) with `rows`
- * token rows and the adapter rows on or off, back to back on the context's stream.  Successive
- * launches read different layers' weights (larger than L2 in total).  *h_ms_per_launch receives
- * the mean launch duration from CUDA events; *h_weight_bytes the weight bytes one launch reads.
- * Buffers hold whatever the last pass left; only the timing is meaningful. */
-pbd_status pbd_time_linear(pbd_ctx *ctx, int32_t which, int32_t rows, int32_t adapter, int32_t iters,
-                           double *h_ms_per_launch, double *h_weight_bytes);
+/* Times the persistent pass kernel alone (all decoder layers of one pass; the lm_head and the
+ * small kernels around it excluded).  On a prefilled context, launches the draft (kind 0),
+ * verify (1) or plain-decoding (2) pass kernel `iters` times with CUDA events bracketing each
+ * launch; the decoding state is not advanced, so every launch does the same work, and the
+ * weights it streams (about 0.9 GB for the 0.6B shape) exceed L2.  *h_ms_per_launch receives the
+ * mean duration; *h_bytes_per_launch the algorithmic bytes of one launch: every layer weight once
+ * (adapter factors too for the draft), the cached K/V read and the block's K/V written. */
+pbd_status pbd_time_pass(pbd_ctx *ctx, int32_t kind, int32_t iters, double *h_ms_per_launch,
+                         double *h_bytes_per_launch);
 
 const char *pbd_last_error(const pbd_ctx *ctx);
 

@@ -24,6 +24,7 @@ enum : int {
     DEV_TIMEOUT_SLOT = 3,   // a ring slot was never released
     DEV_BAD_TOKEN = 4,      // token id outside [0, V)
     DEV_BAD_POSITION = 5,   // position beyond the reserved pages
+    DEV_TIMEOUT_DEP = 6,    // a work item's inputs never completed
 };
 
 constexpr unsigned long long WAIT_LIMIT_NS = 1000000000ull;  // 1 s
@@ -60,6 +61,10 @@ __device__ __forceinline__ void fence_mbarrier_init() {
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
                  : "memory");
+}
+
+__device__ __forceinline__ void mbarrier_arrive_one(uint64_t *bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {

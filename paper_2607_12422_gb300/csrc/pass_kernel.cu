@@ -1,0 +1,991 @@
+// pass_kernel.cu -- one persistent, cooperative kernel per decoder pass (draft, verify, plain
+// decoding, prefill chunk) of the PEFT-BD hot path.
+//
+// Why: at batch 1 and D = 16 a pass moves 1.2 GB of weights (~180 us at full HBM bandwidth)
+// through ~500 small dependent steps.  As separate kernel launches, launch gaps and latency
+// chains dominated.  Here one CTA per SM walks a static, topologically ordered list of work
+// items, and items wait only for the items they read (per-tile counters in global memory with
+// bounded spins), so phases overlap and no kernel boundary separates them.
+//
+// Roles inside a CTA (256 threads):
+//   warp 0      weight producer: walks the CTA's linear items ahead of the others and streams
+//               their 128 x 64 weight tiles (16 KiB, pre-tiled in the 128-byte swizzle layout)
+//               into a ring of shared-memory slots with 1-D bulk TMA (L2 evict-first).  Weights
+//               depend on nothing, so the ring fills across phase boundaries.
+//   warp 1      MMA issuer: per linear item, 4 x 4 tcgen05.mma (128 x BN x 16, bf16 -> fp32) into
+//               a TMEM accumulator; frees ring slots with tcgen05.commit.
+//   warps 2-7   compute group: dependency waits, operand staging (RMSNorm applied on the fly
+//               while building the activation tile in the swizzle layout), the TMEM epilogue
+//               (warps 4-7, one per TMEM lane quarter), attention, split reductions.
+//
+// A linear is split along K into 256-wide slices (fixed per linear, independent of the row
+// count).  Each slice item stores fp32 partial sums; the CTA that completes a tile last (atomic
+// counter) adds the slices in slice order and finishes the step for that tile:
+//   q|k|v tile   -> + adapter delta, bf16, per-head RMSNorm, RoPE, q buffer / paged K, V
+//   o tile       -> + adapter delta, residual add into h, per-tile sum of squares of h
+//   gate|up tile -> + adapter delta, SiLU(gate) * up into the act buffer (gate/up interleaved)
+//   down tile    -> + adapter delta, residual add into h, per-tile sum of squares of h
+//   adapter tile -> u = bf16(x A^T) for the tiles above (scheduled first in every phase)
+// Attention items cover (sequence, KV head, 128-key split); the last split of a head group
+// merges the splits into the attention output.  RMSNorm statistics are summed per 128-feature
+// tile in one fixed order, so every row's arithmetic is independent of the pass it is in.
+#include <algorithm>
+#include <cmath>
+#include <vector>
+
+#include "common.cuh"
+#include "pbd_internal.h"
+
+namespace pbd {
+
+constexpr int MK_THREADS = 256;
+constexpr int CT = 192;            // compute-group threads (warps 2-7)
+constexpr int KSLICE = 256;        // K elements per linear item
+constexpr int ATOMS = KSLICE / KT; // 64-wide swizzle atoms per item
+constexpr int MAX_SLOT = 12;
+constexpr int MAX_ROWS = 256;
+
+// ------------------------------------------------------------------ device helpers
+
+__device__ __forceinline__ void bar_compute() { asm volatile("bar.sync 1, 192;" ::: "memory"); }
+
+__device__ __forceinline__ int ld_acquire(const int *p) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ int ld_relaxed(const int *p) {
+    int v;
+    asm volatile("ld.relaxed.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+struct MKParams {
+    Dims dm;
+    PassDesc pd;
+    const MKItem *items;
+    const int *cta_off;
+    int *cnt;            // counters of this pass (zeroed before launch)
+    CounterLayout cl;
+    const int *nsplit;   // [nb] attention split items per sequence
+    // weights
+    const uint8_t *wt[4];      // tiled weights of layer 0; layer stride wt_stride[lin] bytes
+    size_t wt_stride[4];
+    int n_main[4], lora_rows[4], K[4], ks[4];
+    const bf16 *lora_b[4];     // fused adapter B of layer 0, [n_out][r]
+    size_t lb_stride[4];       // elements per layer
+    const bf16 *attn_norm, *mlp_norm, *q_norm, *k_norm, *final_norm, *mask_embed, *embed_tiled;
+    const float2 *rope_cs;
+    int rope_rows;
+    KVCache kv;
+    const int *L;
+    const int *ids;
+    // scratch
+    float *part[4];
+    int part_rows;
+    float *red_lora[4];
+    bf16 *h, *q, *attn, *act, *x_ro;
+    float *ss;                 // [rows][H/128]
+    float *o_part;
+    float2 *ml_part;
+    int att_splits_alloc;
+    float att_scale;           // 1/sqrt(head_dim)
+    int *status, *abort;
+    // launch geometry
+    int bn, nslot, ring_bytes, union_bytes;
+    uint32_t tmem_cols;
+};
+
+__device__ __forceinline__ bool aborted(const MKParams &P) { return ld_relaxed(P.abort) != 0; }
+
+__device__ __forceinline__ void raise_abort(const MKParams &P, int code) {
+    latch_error(P.status, code);
+    atomicExch(P.abort, 1);
+}
+
+// one thread: wait until *c >= target (bounded)
+__device__ bool spin_until(const int *c, int target, const MKParams &P) {
+    if (ld_acquire(c) >= target) return true;
+    const uint64_t t0 = globaltimer_ns();
+    for (;;) {
+        for (int i = 0; i < 8; ++i) {
+            if (ld_acquire(c) >= target) return true;
+            __nanosleep(40);
+        }
+        if (aborted(P)) return false;
+        if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
+            raise_abort(P, DEV_TIMEOUT_DEP);
+            return false;
+        }
+    }
+}
+
+// bounded mbarrier wait that also gives up when the pass is aborted
+__device__ bool mbar_wait_mk(uint64_t *bar, uint32_t parity, const MKParams &P, int code) {
+    const uint32_t a = smem_u32(bar);
+    if (mbar_try_wait(a, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    for (;;) {
+        for (int i = 0; i < 16; ++i)
+            if (mbar_try_wait(a, parity)) return true;
+        if (aborted(P)) return false;
+        if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
+            raise_abort(P, code);
+            return false;
+        }
+    }
+}
+
+__device__ __forceinline__ int *ctr(const MKParams &P, int layer, int off) {
+    return P.cnt + P.cl.global + layer * P.cl.per_layer + off;
+}
+
+// Sum of squares of one 128-feature tile of a row, in one fixed order: lane l adds elements
+// l, l+32, l+64, l+96 in that order, then a butterfly; lane 0's value is the result.
+__device__ __forceinline__ float tile_sumsq(const float (&v)[4]) {
+    float s = __fmul_rn(v[0], v[0]);
+#pragma unroll
+    for (int e = 1; e < 4; ++e) s = __fadd_rn(s, __fmul_rn(v[e], v[e]));
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) s = __fadd_rn(s, __shfl_xor_sync(0xffffffffu, s, off));
+    return __shfl_sync(0xffffffffu, s, 0);
+}
+
+// 1/sqrt(mean(h^2) + eps) of row m from its per-tile sums (tiles added in order)
+__device__ __forceinline__ float row_rms(const MKParams &P, int m) {
+    const int nt = P.dm.H / TILE_ROWS;
+    const float *s = P.ss + (size_t)m * nt;
+    float a = s[0];
+    for (int t = 1; t < nt; ++t) a = __fadd_rn(a, s[t]);
+    return __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(__fdiv_rn(a, (float)P.dm.H), P.dm.eps)));
+}
+
+__device__ __forceinline__ float lora_dot_f(const float *u, const bf16 *Brow, int r) {
+    float a = 0.f;
+    for (int j = 0; j < r; ++j) a = __fadd_rn(a, __fmul_rn(u[j], bf2f(Brow[j])));
+    return a;
+}
+
+__device__ __forceinline__ float sum_part(const MKParams &P, int lin, int m, int f) {
+    const int nt = P.n_main[lin] + P.lora_rows[lin];
+    const float *p = P.part[lin] + (size_t)m * nt + f;
+    const size_t stride = (size_t)P.part_rows * nt;
+    float a = p[0];
+    for (int s = 1; s < P.ks[lin]; ++s) a = __fadd_rn(a, p[s * stride]);
+    return a;
+}
+
+// element (v, k) of a matrix in the 128 x 64 swizzled tile layout
+__device__ __forceinline__ const bf16 *tiled_at(const bf16 *tiles, int K, int v, int k) {
+    const int t = v >> 7, r = v & 127, kt = k >> 6, c = (k & 63) >> 3, e = k & 7;
+    return tiles + ((size_t)t * (K >> 6) + kt) * (TILE_ROWS * KT) + r * KT + ((c ^ (r & 7)) << 3) + e;
+}
+
+// ------------------------------------------------------------------ work items
+
+// token / mask-embedding row -> residual h and its per-tile sums of squares
+__device__ void do_embed(const MKParams &P, int m, int cw, int lane) {
+    int tok = P.ids[m];
+    if (tok >= P.dm.V) {
+        latch_error(P.status, DEV_BAD_TOKEN);
+        tok = 0;
+    }
+    const int H = P.dm.H, nt = H / TILE_ROWS;
+    for (int t = cw; t < nt; t += CT / 32) {
+        float v[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int f = t * TILE_ROWS + lane + 32 * e;
+            v[e] = tok >= 0 ? bf2f(*tiled_at(P.embed_tiled, H, tok, f)) : bf2f(P.mask_embed[f]);
+            P.h[(size_t)m * H + f] = f2bf(v[e]);
+        }
+        const float s = tile_sumsq(v);
+        if (lane == 0) P.ss[(size_t)m * nt + t] = s;
+    }
+}
+
+// Activation tile of one linear item in the 128-byte swizzle layout: atom j (K columns
+// 64j..64j+63 of the slice) holds row m at m*128 bytes, 16-byte chunk c at (c ^ (m & 7)) * 16.
+__device__ void build_b(const MKParams &P, int lin, int layer, int slice, uint8_t *sb, float *s_rms, int ct) {
+    const int M = P.pd.M;
+    const int k0 = slice * KSLICE;
+    const bool norm = (lin == 0 || lin == 2);
+    if (norm) {
+        for (int m = ct; m < M; m += CT) s_rms[m] = row_rms(P, m);
+        bar_compute();
+    }
+    const bf16 *gain = lin == 0 ? P.attn_norm + (size_t)layer * P.dm.H : P.mlp_norm + (size_t)layer * P.dm.H;
+    const int chunks = M * (KSLICE / 8);
+    for (int q = ct; q < chunks; q += CT) {
+        const int m = q / (KSLICE / 8), c = q % (KSLICE / 8);
+        const int atom = c >> 3, cc = c & 7;
+        uint4 val;
+        if (norm) {
+            const uint4 hv = *reinterpret_cast<const uint4 *>(P.h + (size_t)m * P.dm.H + k0 + c * 8);
+            const uint4 gv = *reinterpret_cast<const uint4 *>(gain + k0 + c * 8);
+            const bf16 *he = reinterpret_cast<const bf16 *>(&hv);
+            const bf16 *ge = reinterpret_cast<const bf16 *>(&gv);
+            bf16 *oe = reinterpret_cast<bf16 *>(&val);
+            const float rs = s_rms[m];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) oe[e] = f2bf(__fmul_rn(bf2f(ge[e]), rbf(__fmul_rn(bf2f(he[e]), rs))));
+        } else {
+            const bf16 *src = lin == 1 ? P.attn + (size_t)m * (P.dm.Hq * P.dm.d) : P.act + (size_t)m * P.dm.I;
+            val = *reinterpret_cast<const uint4 *>(src + k0 + c * 8);
+        }
+        *reinterpret_cast<uint4 *>(sb + (size_t)atom * P.bn * 128 + m * 128 + ((cc ^ (m & 7)) << 4)) = val;
+    }
+}
+
+// reducer of the adapter tile: u = bf16(sum of slices), kept as fp32 values
+__device__ void reduce_lora(const MKParams &P, int lin, int ct) {
+    const int M = P.pd.M, lr = P.lora_rows[lin], n0 = P.n_main[lin];
+    for (int q = ct; q < M * lr; q += CT) {
+        const int m = q / lr, j = q % lr;
+        P.red_lora[lin][q] = rbf(sum_part(P, lin, m, n0 + j));
+    }
+}
+
+// q|k|v tile: adapter delta, bf16, per-head RMSNorm + RoPE for q and k, store q / paged K, V
+template <int DH>
+__device__ void reduce_qkv(const MKParams &P, int layer, int tile, int cw, int lane) {
+    constexpr int E = DH / 32;
+    const Dims &dm = P.dm;
+    const int M = P.pd.M, r = dm.r;
+    const int heads_per_tile = TILE_ROWS / DH;
+    const bf16 *lb = P.lora_b[0] + (size_t)layer * P.lb_stride[0];
+    for (int it = cw; it < M * heads_per_tile; it += CT / 32) {
+        const int m = it / heads_per_tile, hh = it % heads_per_tile;
+        const int fbase = tile * TILE_ROWS + hh * DH;
+        const int qw = dm.Hq * DH, kvw = dm.Hkv * DH;
+        const int kind = fbase < qw ? 0 : (fbase < qw + kvw ? 1 : 2);
+        const int head = kind == 0 ? fbase / DH : (kind == 1 ? (fbase - qw) / DH : (fbase - qw - kvw) / DH);
+        const int b = P.pd.b0 + m / P.pd.R;
+        const int pos = P.L[b] + m % P.pd.R;
+        const float *u = P.red_lora[0] + (size_t)m * P.lora_rows[0] + kind * r;
+        float y[E];
+#pragma unroll
+        for (int j = 0; j < E; ++j) {
+            const int f = fbase + lane + 32 * j;
+            float acc = sum_part(P, 0, m, f);
+            if (P.pd.adapter) acc = __fadd_rn(acc, __fmul_rn(dm.lora_scale, lora_dot_f(u, lb + (size_t)f * r, r)));
+            y[j] = rbf(acc);
+        }
+        if (kind < 2) {
+            const bf16 *gn = (kind == 0 ? P.q_norm : P.k_norm) + (size_t)layer * DH;
+            float ss = 0.f;
+#pragma unroll
+            for (int j = 0; j < E; ++j) ss = __fadd_rn(ss, __fmul_rn(y[j], y[j]));
+#pragma unroll
+            for (int off = 16; off >= 1; off >>= 1) ss = __fadd_rn(ss, __shfl_xor_sync(0xffffffffu, ss, off));
+            ss = __shfl_sync(0xffffffffu, ss, 0);
+            const float rs = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(__fdiv_rn(ss, (float)DH), dm.eps)));
+#pragma unroll
+            for (int j = 0; j < E; ++j) y[j] = rbf(__fmul_rn(bf2f(gn[lane + 32 * j]), rbf(__fmul_rn(y[j], rs))));
+            if (pos >= P.rope_rows) {
+                latch_error(P.status, DEV_BAD_POSITION);
+                continue;
+            }
+#pragma unroll
+            for (int j = 0; j < E / 2; ++j) {
+                const int e = lane + 32 * j;
+                const float2 cs = P.rope_cs[(size_t)pos * (DH / 2) + e];
+                const float a = y[j], c = y[j + E / 2];
+                y[j] = rbf(__fsub_rn(__fmul_rn(a, cs.x), __fmul_rn(c, cs.y)));
+                y[j + E / 2] = rbf(__fadd_rn(__fmul_rn(c, cs.x), __fmul_rn(a, cs.y)));
+            }
+        }
+        if (kind == 0) {
+            bf16 *dst = P.q + ((size_t)m * dm.Hq + head) * DH;
+#pragma unroll
+            for (int j = 0; j < E; ++j) dst[lane + 32 * j] = f2bf(y[j]);
+        } else {
+            const int pg = pos / PAGE;
+            if (pg >= P.kv.pages_per_seq) {
+                latch_error(P.status, DEV_BAD_POSITION);
+                continue;
+            }
+            const int page = P.kv.page_table[b * P.kv.pages_per_seq + pg];
+            const size_t off = ((((size_t)layer * P.kv.n_pages + page) * dm.Hkv + head) * PAGE + (pos % PAGE)) * DH;
+            bf16 *dst = static_cast<bf16 *>(kind == 1 ? P.kv.k : P.kv.v) + off;
+#pragma unroll
+            for (int j = 0; j < E; ++j) dst[lane + 32 * j] = f2bf(y[j]);
+        }
+    }
+}
+
+// o or down tile: adapter delta, residual add into h, per-tile sum of squares
+__device__ void reduce_residual(const MKParams &P, int lin, int layer, int tile, int cw, int lane) {
+    const Dims &dm = P.dm;
+    const int M = P.pd.M, r = dm.r, H = dm.H, nt = H / TILE_ROWS;
+    const bf16 *lb = P.lora_b[lin] + (size_t)layer * P.lb_stride[lin];
+    for (int m = cw; m < M; m += CT / 32) {
+        const float *u = P.red_lora[lin] + (size_t)m * P.lora_rows[lin];
+        float v[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int f = tile * TILE_ROWS + lane + 32 * e;
+            float acc = sum_part(P, lin, m, f);
+            if (P.pd.adapter) acc = __fadd_rn(acc, __fmul_rn(dm.lora_scale, lora_dot_f(u, lb + (size_t)f * r, r)));
+            const float y = rbf(acc);
+            const float hn = rbf(__fadd_rn(bf2f(P.h[(size_t)m * H + f]), y));
+            P.h[(size_t)m * H + f] = f2bf(hn);
+            v[e] = hn;
+        }
+        const float s = tile_sumsq(v);
+        if (lane == 0) P.ss[(size_t)m * nt + tile] = s;
+    }
+}
+
+// gate|up tile (rows 0-63 gate features 64t.., rows 64-127 up features 64t..): SiLU(gate)*up
+__device__ void reduce_gu(const MKParams &P, int layer, int tile, int cw, int lane) {
+    const Dims &dm = P.dm;
+    const int M = P.pd.M, r = dm.r, I = dm.I;
+    const bf16 *lb = P.lora_b[2] + (size_t)layer * P.lb_stride[2];
+    for (int m = cw; m < M; m += CT / 32) {
+        const float *u = P.red_lora[2] + (size_t)m * P.lora_rows[2];
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            const int j = lane + 32 * e;  // 0..63
+            const int f = tile * 64 + j;  // act feature
+            float g = sum_part(P, 2, m, tile * TILE_ROWS + j);
+            float up = sum_part(P, 2, m, tile * TILE_ROWS + 64 + j);
+            if (P.pd.adapter) {
+                g = __fadd_rn(g, __fmul_rn(dm.lora_scale, lora_dot_f(u, lb + (size_t)f * r, r)));
+                up = __fadd_rn(up, __fmul_rn(dm.lora_scale, lora_dot_f(u + r, lb + (size_t)(I + f) * r, r)));
+            }
+            g = rbf(g);
+            up = rbf(up);
+            const float sg = __fdiv_rn(g, __fadd_rn(1.0f, expf(-g)));
+            P.act[(size_t)m * I + f] = f2bf(__fmul_rn(sg, up));
+        }
+    }
+}
+
+// ---- attention: one (sequence, KV head, 128-key split) on the compute group
+
+__device__ __forceinline__ uint32_t ldu32(const void *p) { return *reinterpret_cast<const uint32_t *>(p); }
+
+template <int DH>
+__device__ void attn_split(const MKParams &P, int layer, int bl, int g, int s, uint8_t *smem, int ct, int cw,
+                           int lane) {
+    constexpr int KSTR = DH + 8, VSTR = DH + 8;
+    constexpr int NT = ATT_SPLIT / 8, KS = DH / 16, DT = DH / 8;
+    const Dims &dm = P.dm;
+    const int b = P.pd.b0 + bl;
+    const int L = P.L[b];
+    const int R = P.pd.R;
+    const int T = L + R;
+    const int k0 = s * ATT_SPLIT;
+    const int grp = dm.Hq / dm.Hkv;
+    const int QV = R * grp;
+    const int n_mt = (QV + 15) / 16;
+    bf16 *sK = reinterpret_cast<bf16 *>(smem);
+    __half *sV = reinterpret_cast<__half *>(smem + ATT_SPLIT * KSTR * 2);
+    const size_t layer_off = (size_t)layer * P.kv.n_pages * dm.Hkv * PAGE * DH;
+    const bf16 *kc = static_cast<const bf16 *>(P.kv.k), *vc = static_cast<const bf16 *>(P.kv.v);
+    for (int idx = ct; idx < ATT_SPLIT * (DH / 8); idx += CT) {
+        const int kk = idx / (DH / 8), c = idx % (DH / 8);
+        const int kp = k0 + kk;
+        uint4 k4 = make_uint4(0, 0, 0, 0), v4 = make_uint4(0, 0, 0, 0);
+        if (kp < T && kp / PAGE < P.kv.pages_per_seq) {
+            const int page = P.kv.page_table[b * P.kv.pages_per_seq + kp / PAGE];
+            const size_t off = layer_off + (((size_t)page * dm.Hkv + g) * PAGE + (kp % PAGE)) * DH + (size_t)c * 8;
+            k4 = *reinterpret_cast<const uint4 *>(kc + off);
+            v4 = *reinterpret_cast<const uint4 *>(vc + off);
+        }
+        *reinterpret_cast<uint4 *>(sK + kk * KSTR + c * 8) = k4;
+        const bf16 *ve = reinterpret_cast<const bf16 *>(&v4);
+        uint4 h4;
+        uint32_t *hw = reinterpret_cast<uint32_t *>(&h4);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) hw[e] = pack_half2(bf2f(ve[2 * e]), bf2f(ve[2 * e + 1]));
+        *reinterpret_cast<uint4 *>(sV + kk * VSTR + c * 8) = h4;
+    }
+    bar_compute();
+    const int gq = lane >> 2, tq = lane & 3;
+    const bool blk = P.pd.mask_mode == MASK_BLOCK_DRAFT;
+    for (int mt = cw; mt < n_mt; mt += CT / 32) {
+        const int qv0 = mt * 16 + gq, qv1 = qv0 + 8;
+        const bool val0 = qv0 < QV, val1 = qv1 < QV;
+        const int i0 = val0 ? qv0 / grp : 0, i1 = val1 ? qv1 / grp : 0;
+        const int h0 = g * grp + (val0 ? qv0 % grp : 0), h1 = g * grp + (val1 ? qv1 % grp : 0);
+        const bf16 *q0 = P.q + ((size_t)(bl * R + i0) * dm.Hq + h0) * DH;
+        const bf16 *q1 = P.q + ((size_t)(bl * R + i1) * dm.Hq + h1) * DH;
+        uint32_t qa[KS][4];
+#pragma unroll
+        for (int ks = 0; ks < KS; ++ks) {
+            const int c = ks * 16 + 2 * tq;
+            qa[ks][0] = val0 ? ldu32(q0 + c) : 0u;
+            qa[ks][1] = val1 ? ldu32(q1 + c) : 0u;
+            qa[ks][2] = val0 ? ldu32(q0 + c + 8) : 0u;
+            qa[ks][3] = val1 ? ldu32(q1 + c + 8) : 0u;
+        }
+        float sc[NT][4];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+            sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
+            const bf16 *krow = sK + (nt * 8 + gq) * KSTR + 2 * tq;
+#pragma unroll
+            for (int ks = 0; ks < KS; ++ks) mma_m16n8k16_bf16(sc[nt], qa[ks], ldu32(krow + ks * 16), ldu32(krow + ks * 16 + 8));
+        }
+        const int qp0 = L + i0, qp1 = L + i1;
+        const float scale = P.att_scale;
+        float m0 = -INFINITY, m1 = -INFINITY;
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const int kp = k0 + nt * 8 + 2 * tq + e;
+                const bool vis0 = val0 && kp < T && (kp <= qp0 || (blk && i0 >= 1 && kp > L));
+                const bool vis1 = val1 && kp < T && (kp <= qp1 || (blk && i1 >= 1 && kp > L));
+                sc[nt][e] = vis0 ? __fmul_rn(sc[nt][e], scale) : -INFINITY;
+                sc[nt][2 + e] = vis1 ? __fmul_rn(sc[nt][2 + e], scale) : -INFINITY;
+                m0 = fmaxf(m0, sc[nt][e]);
+                m1 = fmaxf(m1, sc[nt][2 + e]);
+            }
+        }
+        m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, 1));
+        m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, 2));
+        m1 = fmaxf(m1, __shfl_xor_sync(0xffffffffu, m1, 1));
+        m1 = fmaxf(m1, __shfl_xor_sync(0xffffffffu, m1, 2));
+        const float mz0 = m0 == -INFINITY ? 0.f : m0, mz1 = m1 == -INFINITY ? 0.f : m1;
+        float l0 = 0.f, l1 = 0.f;
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const float p0 = sc[nt][e] == -INFINITY ? 0.f : __expf(sc[nt][e] - mz0);
+                const float p1 = sc[nt][2 + e] == -INFINITY ? 0.f : __expf(sc[nt][2 + e] - mz1);
+                sc[nt][e] = p0;
+                sc[nt][2 + e] = p1;
+                l0 += p0;
+                l1 += p1;
+            }
+        }
+        l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+        l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+        l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+        l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+        float oc[DT][4];
+#pragma unroll
+        for (int dt = 0; dt < DT; ++dt) oc[dt][0] = oc[dt][1] = oc[dt][2] = oc[dt][3] = 0.f;
+#pragma unroll
+        for (int kstep = 0; kstep < ATT_SPLIT / 16; ++kstep) {
+            uint32_t pa[4];
+            pa[0] = pack_half2(sc[2 * kstep][0], sc[2 * kstep][1]);
+            pa[1] = pack_half2(sc[2 * kstep][2], sc[2 * kstep][3]);
+            pa[2] = pack_half2(sc[2 * kstep + 1][0], sc[2 * kstep + 1][1]);
+            pa[3] = pack_half2(sc[2 * kstep + 1][2], sc[2 * kstep + 1][3]);
+            const int vrow = kstep * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+#pragma unroll
+            for (int dt = 0; dt < DT; dt += 2) {
+                const int vcol = dt * 8 + (lane >> 4) * 8;
+                const uint32_t addr = smem_u32(sV + vrow * VSTR + vcol);
+                uint32_t r0, r1, r2, r3;
+                asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                             : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                             : "r"(addr));
+                mma_m16n8k16_f16(oc[dt], pa, r0, r1);
+                mma_m16n8k16_f16(oc[dt + 1], pa, r2, r3);
+            }
+        }
+        const int nsa = P.att_splits_alloc;
+        if (val0) {
+            const int m = bl * R + i0;
+            float *dst = P.o_part + (((size_t)m * dm.Hq + h0) * nsa + s) * DH;
+#pragma unroll
+            for (int dt = 0; dt < DT; ++dt)
+                *reinterpret_cast<float2 *>(dst + dt * 8 + 2 * tq) = make_float2(oc[dt][0], oc[dt][1]);
+            if (tq == 0) P.ml_part[((size_t)m * dm.Hq + h0) * nsa + s] = make_float2(m0, l0);
+        }
+        if (val1) {
+            const int m = bl * R + i1;
+            float *dst = P.o_part + (((size_t)m * dm.Hq + h1) * nsa + s) * DH;
+#pragma unroll
+            for (int dt = 0; dt < DT; ++dt)
+                *reinterpret_cast<float2 *>(dst + dt * 8 + 2 * tq) = make_float2(oc[dt][2], oc[dt][3]);
+            if (tq == 0) P.ml_part[((size_t)m * dm.Hq + h1) * nsa + s] = make_float2(m1, l1);
+        }
+    }
+}
+
+// merge the splits of (row, head) in split order; splits where the row saw no key are skipped
+template <int DH>
+__device__ void attn_combine(const MKParams &P, int bl, int g, int cw, int lane) {
+    const Dims &dm = P.dm;
+    const int R = P.pd.R, grp = dm.Hq / dm.Hkv;
+    const int b = P.pd.b0 + bl;
+    const int T = P.L[b] + R;
+    const int nsa = P.att_splits_alloc;
+    const int nv = min(P.nsplit[bl], (T + ATT_SPLIT - 1) / ATT_SPLIT);  // splits computed in this pass
+    constexpr int E = DH / 32;
+    for (int it = cw; it < R * grp; it += CT / 32) {
+        const int i = it / grp, h = g * grp + it % grp;
+        const int m = bl * R + i;
+        const float2 *ml = P.ml_part + ((size_t)m * dm.Hq + h) * nsa;
+        float mx = -INFINITY;
+        for (int s = 0; s < nv; ++s) {
+            const float2 v = ml[s];
+            if (v.y > 0.f) mx = fmaxf(mx, v.x);
+        }
+        float num[E];
+#pragma unroll
+        for (int e = 0; e < E; ++e) num[e] = 0.f;
+        float den = 0.f;
+        for (int s = 0; s < nv; ++s) {
+            const float2 v = ml[s];
+            if (!(v.y > 0.f)) continue;
+            const float w = __expf(v.x - mx);
+            den = __fadd_rn(den, __fmul_rn(w, v.y));
+            const float *o = P.o_part + (((size_t)m * dm.Hq + h) * nsa + s) * DH;
+#pragma unroll
+            for (int e = 0; e < E; ++e) num[e] = __fadd_rn(num[e], __fmul_rn(w, o[lane + 32 * e]));
+        }
+        bf16 *dst = P.attn + ((size_t)m * dm.Hq + h) * DH;
+#pragma unroll
+        for (int e = 0; e < E; ++e) dst[lane + 32 * e] = f2bf(__fdiv_rn(num[e], den));
+    }
+}
+
+// wait for every tile of linear `lin` that holds output features [f0, f1)
+__device__ bool wait_tiles(const MKParams &P, int layer, int lin, int f0, int f1) {
+    const int off = P.cl.lin[lin];
+    for (int t = f0 / TILE_ROWS; t <= (f1 - 1) / TILE_ROWS; ++t)
+        if (!spin_until(ctr(P, layer, off + t), P.ks[lin] + 1, P)) return false;
+    return true;
+}
+
+// the item's inputs are complete (one thread; false on abort)
+__device__ bool wait_deps(const MKParams &P, const MKItem &it) {
+    const Dims &dm = P.dm;
+    const int l = it.layer;
+    if (it.op == MK_LINEAR) {
+        const int s = it.b;
+        switch (it.lin) {
+            case 0:
+                if (l == 0) return spin_until(P.cnt + P.cl.embed, P.pd.M, P);
+                return spin_until(ctr(P, l - 1, P.cl.res_dn), dm.H / TILE_ROWS, P);
+            case 1: {
+                const int h0 = (s * KSLICE) / dm.d, h1 = (s * KSLICE + KSLICE - 1) / dm.d;
+                const int grp = dm.Hq / dm.Hkv;
+                for (int bl = 0; bl < P.pd.nb; ++bl)
+                    for (int g = h0 / grp; g <= h1 / grp; ++g)
+                        if (!spin_until(ctr(P, l, P.cl.att + bl * dm.Hkv + g), P.nsplit[bl] + 1, P)) return false;
+                return true;
+            }
+            case 2: return spin_until(ctr(P, l, P.cl.res_o), dm.H / TILE_ROWS, P);
+            default: {
+                // act features [256 s, 256 s + 256) live in gate|up tiles 4s..4s+3
+                const int t0 = (s * KSLICE) / 64, t1 = (s * KSLICE + KSLICE - 1) / 64;
+                for (int t = t0; t <= t1; ++t)
+                    if (!spin_until(ctr(P, l, P.cl.lin[2] + t), P.ks[2] + 1, P)) return false;
+                return true;
+            }
+        }
+    }
+    if (it.op == MK_ATTN) {
+        const int g = it.b, grp = dm.Hq / dm.Hkv, d = dm.d;
+        const int qw = dm.Hq * d, kvw = dm.Hkv * d;
+        return wait_tiles(P, l, 0, g * grp * d, (g + 1) * grp * d) &&
+               wait_tiles(P, l, 0, qw + g * d, qw + (g + 1) * d) &&
+               wait_tiles(P, l, 0, qw + kvw + g * d, qw + kvw + (g + 1) * d);
+    }
+    if (it.op == MK_FINAL) return spin_until(ctr(P, dm.nl - 1, P.cl.res_dn), dm.H / TILE_ROWS, P);
+    return true;
+}
+
+// ------------------------------------------------------------------ the kernel
+
+__global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ MKParams P) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *ring = base;
+    uint8_t *uni = base + P.ring_bytes;  // activation tile / attention staging
+    __shared__ __align__(8) uint64_t full[MAX_SLOT], empty[MAX_SLOT], b_full, acc_full;
+    __shared__ uint32_t tmem_slot;
+    // compute-group flags: each is written by thread 0 and read by all after a barrier, and is
+    // not written again before every thread has passed at least one more barrier
+    __shared__ int s_flag, s_red, s_ok;
+    __shared__ float s_rms[MAX_ROWS];
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const MKItem *my = P.items + P.cta_off[blockIdx.x];
+    const int n_my = P.cta_off[blockIdx.x + 1] - P.cta_off[blockIdx.x];
+
+    if (tid == 0) {
+        for (int i = 0; i < P.nslot; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
+        mbar_init(&b_full, 1);
+        mbar_init(&acc_full, 1);
+        fence_mbarrier_init();
+    }
+    if (warp == 0) tmem_alloc(&tmem_slot, P.tmem_cols);
+    // zero the padding rows of the activation tile once (rows >= M are never written)
+    for (int q = tid; q < ATOMS * P.bn * 8; q += MK_THREADS) {
+        const int atom = q / (P.bn * 8), rem = q % (P.bn * 8), m = rem / 8;
+        if (m >= P.pd.M) *reinterpret_cast<uint4 *>(uni + (size_t)atom * P.bn * 128 + rem * 16) = make_uint4(0, 0, 0, 0);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+
+    if (warp == 0) {
+        // ---------------- weight producer
+        if (lane == 0) {
+            const uint64_t pol = l2_policy_evict_first();
+            uint32_t kt = 0;
+            for (int i = 0; i < n_my && !aborted(P); ++i) {
+                const MKItem it = my[i];
+                if (it.op != MK_LINEAR) continue;
+                const int lin = it.lin;
+                const bool lt = it.a >= P.n_main[lin] / TILE_ROWS;
+                const uint32_t bytes = lt ? (uint32_t)P.lora_rows[lin] * 128u : (uint32_t)TILE_BYTES;
+                const int kts = P.K[lin] / KT;
+                const uint8_t *src = P.wt[lin] + P.wt_stride[lin] * it.layer +
+                                     ((size_t)it.a * kts + (size_t)it.b * ATOMS) * TILE_BYTES;
+                bool ok = true;
+                for (int j = 0; j < ATOMS; ++j, ++kt) {
+                    const int slot = kt % P.nslot;
+                    if (kt >= (uint32_t)P.nslot &&
+                        !mbar_wait_mk(&empty[slot], ((kt / P.nslot) - 1) & 1, P, DEV_TIMEOUT_SLOT)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&full[slot], bytes);
+                    bulk_g2s(ring + (size_t)slot * TILE_BYTES, src + (size_t)j * TILE_BYTES, bytes, &full[slot], pol);
+                }
+                if (!ok) break;
+            }
+        }
+    } else if (warp == 1) {
+        // ---------------- MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16_f32(128, P.bn);
+            uint32_t kt = 0, li = 0;
+            for (int i = 0; i < n_my; ++i) {
+                const MKItem it = my[i];
+                if (it.op != MK_LINEAR) continue;
+                if (!mbar_wait_mk(&b_full, li & 1, P, DEV_TIMEOUT_LOAD)) break;
+                tc_fence_after();
+                bool ok = true;
+                for (int j = 0; j < ATOMS; ++j, ++kt) {
+                    const int slot = kt % P.nslot;
+                    if (!mbar_wait_mk(&full[slot], (kt / P.nslot) & 1, P, DEV_TIMEOUT_LOAD)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint64_t ad = sw128_kmajor_desc(ring + (size_t)slot * TILE_BYTES);
+                    const uint64_t bd = sw128_kmajor_desc(uni + (size_t)j * P.bn * 128);
+#pragma unroll
+                    for (int kk = 0; kk < KT / 16; ++kk)
+                        mma_bf16_ss(tmem, ad + 2ull * kk, bd + 2ull * kk, idesc, (j | kk) != 0 ? 1u : 0u);
+                    mma_commit(&empty[slot]);
+                }
+                if (!ok) break;
+                mma_commit(&acc_full);
+                ++li;
+            }
+        }
+    } else {
+        // ---------------- compute group (warps 2-7)
+        const int ct = tid - 64, cw = warp - 2;
+        uint32_t li = 0;
+        for (int i = 0; i < n_my; ++i) {
+            const MKItem it = my[i];
+            if (ct == 0) s_flag = wait_deps(P, it) ? 1 : 0;
+            bar_compute();
+            if (!s_flag) break;
+            if (it.op == MK_EMBED) {
+                do_embed(P, it.a, cw, lane);
+                bar_compute();
+                if (ct == 0) {
+                    __threadfence();
+                    atomicAdd(P.cnt + P.cl.embed, 1);
+                }
+            } else if (it.op == MK_FINAL) {
+                const int r = it.a, m = it.b;
+                if (ct == 0) s_rms[0] = row_rms(P, m);
+                bar_compute();
+                const float rs = s_rms[0];
+                for (int f = ct; f < P.dm.H; f += CT)
+                    P.x_ro[(size_t)r * P.dm.H + f] =
+                        f2bf(__fmul_rn(bf2f(P.final_norm[f]), rbf(__fmul_rn(bf2f(P.h[(size_t)m * P.dm.H + f]), rs))));
+            } else if (it.op == MK_ATTN) {
+                const int bl = it.a, g = it.b, s = it.c;
+                const int b = P.pd.b0 + bl;
+                if (s * ATT_SPLIT < P.L[b] + P.pd.R) {
+                    if (P.dm.d == 128)
+                        attn_split<128>(P, it.layer, bl, g, s, uni, ct, cw, lane);
+                    else
+                        attn_split<64>(P, it.layer, bl, g, s, uni, ct, cw, lane);
+                }
+                bar_compute();
+                int *c = ctr(P, it.layer, P.cl.att + bl * P.dm.Hkv + g);
+                if (ct == 0) {
+                    __threadfence();
+                    const int old = atomicAdd(c, 1);
+                    __threadfence();
+                    s_red = (old == P.nsplit[bl] - 1) ? 1 : 0;
+                }
+                bar_compute();
+                if (s_red) {
+                    if (P.dm.d == 128)
+                        attn_combine<128>(P, bl, g, cw, lane);
+                    else
+                        attn_combine<64>(P, bl, g, cw, lane);
+                    bar_compute();
+                    if (ct == 0) {
+                        __threadfence();
+                        atomicAdd(c, 1);
+                    }
+                }
+            } else {
+                // ---- linear slice item: stage activations, MMA (warp 1), epilogue, split reduction
+                const int lin = it.lin, l = it.layer, t = it.a, s = it.b;
+                build_b(P, lin, l, s, uni, s_rms, ct);
+                fence_proxy_async();
+                bar_compute();
+                if (ct == 0) mbarrier_arrive_one(&b_full);
+                const bool lt = t >= P.n_main[lin] / TILE_ROWS;
+                const int rows_valid = lt ? P.lora_rows[lin] : TILE_ROWS;
+                if (warp >= 4) {
+                    const int quarter = warp - 4;
+                    const bool have = mbar_wait_mk(&acc_full, li & 1, P, DEV_TIMEOUT_MMA);
+                    tc_fence_after();
+                    if (have) {
+                        const int row = quarter * 32 + lane;
+                        const int n_total = P.n_main[lin] + P.lora_rows[lin];
+                        for (int c0 = 0; c0 < P.bn && c0 < P.pd.M; c0 += 32) {
+                            uint32_t v[32];
+                            tmem_ld_32cols(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)c0, v);
+                            tmem_ld_wait();
+                            if (row < rows_valid) {
+                                float *dst = P.part[lin] + ((size_t)s * P.part_rows + c0) * n_total + t * TILE_ROWS + row;
+#pragma unroll
+                                for (int j = 0; j < 32; ++j)
+                                    if (c0 + j < P.pd.M) dst[(size_t)j * n_total] = __uint_as_float(v[j]);
+                            }
+                        }
+                    }
+                    tc_fence_before();
+                }
+                ++li;
+                bar_compute();
+                int *c = ctr(P, l, P.cl.lin[lin] + t);
+                if (ct == 0) {
+                    __threadfence();
+                    const int old = atomicAdd(c, 1);
+                    __threadfence();
+                    s_red = (old == P.ks[lin] - 1) ? 1 : 0;
+                }
+                bar_compute();
+                if (s_red) {
+                    // this CTA finished the tile last: reduce the slices and finish the step
+                    if (!lt && P.pd.adapter && P.lora_rows[lin] > 0) {
+                        if (ct == 0)
+                            s_ok = spin_until(ctr(P, l, P.cl.lin[lin] + P.n_main[lin] / TILE_ROWS), P.ks[lin] + 1, P)
+                                       ? 1 : 0;
+                        bar_compute();
+                        if (!s_ok) break;
+                    }
+                    if (lt)
+                        reduce_lora(P, lin, ct);
+                    else if (lin == 0) {
+                        if (P.dm.d == 128)
+                            reduce_qkv<128>(P, l, t, cw, lane);
+                        else
+                            reduce_qkv<64>(P, l, t, cw, lane);
+                    } else if (lin == 2)
+                        reduce_gu(P, l, t, cw, lane);
+                    else
+                        reduce_residual(P, lin, l, t, cw, lane);
+                    bar_compute();
+                    if (ct == 0) {
+                        __threadfence();
+                        atomicAdd(c, 1);
+                        if (!lt && (lin == 1 || lin == 3)) atomicAdd(ctr(P, l, lin == 1 ? P.cl.res_o : P.cl.res_dn), 1);
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, P.tmem_cols);
+}
+
+// ------------------------------------------------------------------ host side
+
+static int g_num_sms = 0, g_smem_optin = 0;
+
+static cudaError_t device_limits() {
+    if (g_num_sms) return cudaSuccess;
+    int dev;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+    return cudaDeviceGetAttribute(&g_smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+}
+
+int mk_grid_size() {
+    return device_limits() == cudaSuccess ? g_num_sms : 0;
+}
+
+void mk_counter_layout(const Dims &dm, int max_nb, CounterLayout *cl) {
+    const int nq = (dm.Hq + 2 * dm.Hkv) * dm.d / TILE_ROWS + 1;
+    const int no = dm.H / TILE_ROWS + 1;
+    const int ng = 2 * dm.I / TILE_ROWS + 1;
+    const int nd = dm.H / TILE_ROWS + 1;
+    cl->embed = 0;
+    cl->global = 4;
+    cl->lin[0] = 0;
+    cl->lin[1] = nq;
+    cl->lin[2] = nq + no;
+    cl->lin[3] = nq + no + ng;
+    cl->res_o = nq + no + ng + nd;
+    cl->res_dn = cl->res_o + 1;
+    cl->att = cl->res_dn + 1;
+    cl->per_layer = cl->att + max_nb * dm.Hkv;
+    cl->total = cl->global + dm.nl * cl->per_layer;
+}
+
+// Topologically ordered item list, dealt round-robin over `grid` CTAs (CTA i takes items
+// i, i+grid, ...), so each CTA's list is in dependency order.  Returns items sorted by CTA.
+void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int> &nsplit, int grid,
+                       std::vector<MKItem> *out, std::vector<int> *off) {
+    std::vector<MKItem> all;
+    auto push = [&](uint8_t op, uint8_t lin, int layer, int a, int b, int c) {
+        MKItem it;
+        it.op = op;
+        it.lin = lin;
+        it.layer = (uint16_t)layer;
+        it.a = a;
+        it.b = b;
+        it.c = c;
+        all.push_back(it);
+    };
+    for (int m = 0; m < pd.M; ++m) push(MK_EMBED, 0, 0, m, 0, 0);
+    const int nq = (dm.Hq + 2 * dm.Hkv) * dm.d / TILE_ROWS;
+    const int n_main[4] = {nq, dm.H / TILE_ROWS, 2 * dm.I / TILE_ROWS, dm.H / TILE_ROWS};
+    const int K[4] = {dm.H, dm.Hq * dm.d, dm.H, dm.I};
+    auto linear = [&](int lin, int l) {
+        const int ks = K[lin] / KSLICE;
+        if (pd.adapter)
+            for (int s = 0; s < ks; ++s) push(MK_LINEAR, lin, l, n_main[lin], s, 0);
+        for (int t = 0; t < n_main[lin]; ++t)
+            for (int s = 0; s < ks; ++s) push(MK_LINEAR, lin, l, t, s, 0);
+    };
+    for (int l = 0; l < dm.nl; ++l) {
+        linear(0, l);
+        for (int bl = 0; bl < pd.nb; ++bl)
+            for (int g = 0; g < dm.Hkv; ++g)
+                for (int s = 0; s < nsplit[bl]; ++s) push(MK_ATTN, 0, l, bl, g, s);
+        linear(1, l);
+        linear(2, l);
+        linear(3, l);
+    }
+    for (int bl = 0; bl < pd.nb; ++bl)
+        for (int i = pd.ro_first; i < pd.ro_first + pd.ro_count; ++i)
+            push(MK_FINAL, 0, dm.nl - 1, bl * pd.ro_count + (i - pd.ro_first), bl * pd.R + i, 0);
+    off->assign(grid + 1, 0);
+    for (size_t i = 0; i < all.size(); ++i) (*off)[i % grid + 1]++;
+    for (int c = 0; c < grid; ++c) (*off)[c + 1] += (*off)[c];
+    out->resize(all.size());
+    std::vector<int> fill(off->begin(), off->end() - 1);
+    for (size_t i = 0; i < all.size(); ++i) (*out)[fill[i % grid]++] = all[i];
+}
+
+size_t mk_union_bytes(int bn, int head_dim) {
+    const size_t b = (size_t)ATOMS * bn * 128;
+    const size_t att = (size_t)ATT_SPLIT * (head_dim + 8) * 2 * 2;
+    return std::max(b, att);
+}
+
+cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
+    cudaError_t e = device_limits();
+    if (e != cudaSuccess) return e;
+    MKParams P;
+    P.dm = L.dm;
+    P.pd = L.pd;
+    P.items = L.items;
+    P.cta_off = L.cta_off;
+    P.cnt = L.cnt;
+    P.cl = L.cl;
+    P.nsplit = L.nsplit;
+    for (int i = 0; i < 4; ++i) {
+        P.wt[i] = static_cast<const uint8_t *>(L.wt[i]);
+        P.wt_stride[i] = L.wt_stride[i];
+        P.n_main[i] = L.n_main[i];
+        P.lora_rows[i] = L.lora_rows[i];
+        P.K[i] = L.K[i];
+        P.ks[i] = L.K[i] / KSLICE;
+        P.lora_b[i] = static_cast<const bf16 *>(L.lora_b[i]);
+        P.lb_stride[i] = L.lb_stride[i];
+        P.part[i] = L.part[i];
+        P.red_lora[i] = L.red_lora[i];
+    }
+    P.attn_norm = static_cast<const bf16 *>(L.attn_norm);
+    P.mlp_norm = static_cast<const bf16 *>(L.mlp_norm);
+    P.q_norm = static_cast<const bf16 *>(L.q_norm);
+    P.k_norm = static_cast<const bf16 *>(L.k_norm);
+    P.final_norm = static_cast<const bf16 *>(L.final_norm);
+    P.mask_embed = static_cast<const bf16 *>(L.mask_embed);
+    P.embed_tiled = static_cast<const bf16 *>(L.embed_tiled);
+    P.rope_cs = L.rope_cs;
+    P.rope_rows = L.rope_rows;
+    P.kv = L.kv;
+    P.L = L.Lbuf;
+    P.ids = L.ids;
+    P.part_rows = L.part_rows;
+    P.h = static_cast<bf16 *>(L.h);
+    P.q = static_cast<bf16 *>(L.q);
+    P.attn = static_cast<bf16 *>(L.attn);
+    P.act = static_cast<bf16 *>(L.act);
+    P.x_ro = static_cast<bf16 *>(L.x_ro);
+    P.ss = L.ss;
+    P.o_part = L.o_part;
+    P.ml_part = L.ml_part;
+    P.att_splits_alloc = L.att_splits_alloc;
+    P.att_scale = (float)(1.0 / std::sqrt((double)L.dm.d));
+    P.status = L.status;
+    P.abort = L.abort;
+    P.bn = ((L.pd.M + 31) / 32) * 32;
+    if (P.bn > MAX_ROWS || L.pd.M > MAX_ROWS) return cudaErrorInvalidValue;
+    P.tmem_cols = 32;
+    while ((int)P.tmem_cols < P.bn) P.tmem_cols <<= 1;
+    const size_t uni = mk_union_bytes(P.bn, L.dm.d);
+    const size_t static_smem = 4096;
+    const long avail = (long)g_smem_optin - (long)uni - 1024 - (long)static_smem;
+    P.nslot = (int)std::min<long>(MAX_SLOT, avail / TILE_BYTES);
+    if (P.nslot < 2) return cudaErrorInvalidValue;
+    P.ring_bytes = P.nslot * TILE_BYTES;
+    P.union_bytes = (int)uni;
+    const size_t dyn = (size_t)P.ring_bytes + uni + 1024;
+    static size_t configured = 0;
+    if (dyn > configured) {
+        e = cudaFuncSetAttribute(k_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+        if (e != cudaSuccess) return e;
+        configured = dyn;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(L.grid);
+    cfg.blockDim = dim3(MK_THREADS);
+    cfg.dynamicSmemBytes = dyn;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k_pass, P);
+}
+
+}  // namespace pbd

@@ -2,11 +2,14 @@
 //
 // One context owns a caller-provided device workspace holding: the weights re-tiled for the
 // tensor-core kernels, the adapter's B matrices, a paged bf16 KV cache, the device-resident
-// decoding state (cached lengths, pending tokens, outputs, done flags), and the scratch of
-// the passes (activations, split-K partial sums, attention partials, lm_head tile maxima).
-// A speculative round (draft pass, verify pass, accept/commit) only reads and writes device
-// memory, so it is captured once as a CUDA graph and replayed; the host looks at the done
-// flags every few rounds.
+// decoding state (cached lengths, pending tokens, outputs, done flags), the work schedules of
+// the persistent pass kernel, and the pass scratch (activations, split-K partial sums,
+// attention partials, completion counters, lm_head tile maxima).
+//
+// A pass is: zero the pass counters, build the rows' token ids, one persistent pass kernel
+// (all decoder layers), the lm_head over the read-out rows, the final argmax.  A speculative
+// round (draft pass, verify pass, accept/commit) only reads and writes device memory, so it is
+// captured once as a CUDA graph and replayed; the host looks at the done flags every few rounds.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -33,8 +36,7 @@ const int BN_CHOICES[N_BN] = {32, 64, 128, 256};
 constexpr int POLL_ROUNDS = 4;
 
 enum Phase { PH_NONE = 0, PH_READY, PH_DRAFTED, PH_VERIFIED };
-enum PassKind { PK_DRAFT = 0, PK_VERIFY = 1, PK_DECODE = 2, PK_PREFILL = 3 };
-enum ActBuf { AB_X = 0, AB_ATTN = 1, AB_ACT = 2, AB_XRO = 3, N_AB = 4 };
+enum PassKind { PK_DRAFT = 0, PK_VERIFY = 1, PK_DECODE = 2, PK_PREFILL = 3, N_PK = 4 };
 
 struct Bump {
     uint8_t *base;
@@ -48,11 +50,6 @@ struct Bump {
     }
 };
 
-int k_splits_for(int K) {
-    const int kt = K / KT;
-    return (kt % 4 == 0) ? kt / 4 : 1;  // 256-wide K slices per CTA when possible
-}
-
 int pick_bn(int M) {
     for (int i = 0; i < N_BN; ++i)
         if (M <= BN_CHOICES[i]) return BN_CHOICES[i];
@@ -65,34 +62,43 @@ int bn_index(int bn) {
     return N_BN - 1;
 }
 
+struct Sched {
+    MKItem *items = nullptr;  // device
+    int *off = nullptr;       // device [grid + 1]
+    int *nsplit = nullptr;    // device [max_batch]
+    bool valid = false;
+};
+
 }  // namespace
 
 struct pbd_ctx {
     pbd_config cfg;
     Dims dm;
     cudaStream_t st;
-    int D, rows_alloc, ro_alloc, out_cap, rope_rows, n_splits, pages_per_seq, n_pages;
+    int D, rows_alloc, ro_alloc, out_cap, rope_rows, n_splits, pages_per_seq, n_pages, grid;
+    size_t items_cap;
     // weights
-    std::vector<TiledWeight> w_qkv, w_o, w_gu, w_down;
+    std::vector<TiledWeight> w[4];  // q|k|v, o, gate|up (interleaved), down
     TiledWeight w_lm;
-    void *lb_qkv, *lb_o, *lb_gu, *lb_down;  // adapter B, fused per layer [nl][out][r]
+    void *lb[4];                    // adapter B, fused per layer [nl][out][r]
     void *attn_norm, *mlp_norm, *q_norm, *k_norm, *final_norm, *mask_embed;
     float2 *rope_cs;
     KVCache kv;
     int *page_table;
     // scratch
-    void *h, *x, *q, *attn, *act, *x_ro;
-    float *part;
-    size_t part_floats;
-    float *o_part;
+    void *h, *q, *attn, *act, *x_ro;
+    float *part[4], *red_lora[4], *ss, *o_part;
     float2 *ml_part;
     float *tile_max;
     int *tile_arg;
-    int *ids, *draft_ids, *verify_ids, *first_id, *status;
+    int *ids, *draft_ids, *verify_ids, *first_id, *status, *cnt;  // cnt[0] = abort flag
+    CounterLayout cl;
+    Sched sched[N_PK];
     SeqState s;
-    CUtensorMap maps[N_AB][N_BN];
+    CUtensorMap maps[N_BN];  // x_ro, per box height
     // host state
     int batch = 0, max_new = 0;
+    std::vector<int> prompt_lens;
     Phase phase = PH_NONE;
     std::string err;
     // graphs of pbd_bench_rounds, reused while batch size and forced table are unchanged
@@ -133,11 +139,15 @@ pbd_status fail(pbd_ctx *c, pbd_status code, const char *fmt, ...) {
         if (e_ != cudaSuccess) return fail(c, PBD_ERR_CUDA, "%s: %s", #expr, cudaGetErrorString(e_)); \
     } while (0)
 
+#define TRY(expr)                    \
+    do {                             \
+        pbd_status s_ = (expr);      \
+        if (s_ != PBD_OK) return s_; \
+    } while (0)
+
 bool valid_config(const pbd_config *cfg, std::string *why) {
-    char b[256];
     auto bad = [&](const char *m) {
-        snprintf(b, sizeof b, "%s", m);
-        *why = b;
+        *why = m;
         return false;
     };
     if (!cfg) return bad("null config");
@@ -147,19 +157,30 @@ bool valid_config(const pbd_config *cfg, std::string *why) {
         return bad("non-positive model dimension");
     if (k.head_dim != 64 && k.head_dim != 128) return bad("head_dim must be 64 or 128");
     if (k.n_q_heads % k.n_kv_heads) return bad("n_q_heads must be a multiple of n_kv_heads");
-    if (k.hidden % 128 || k.hidden > 4096) return bad("hidden must be a multiple of 128, at most 4096");
-    if (((k.n_q_heads + 2 * k.n_kv_heads) * k.head_dim) % 128 || (k.n_q_heads * k.head_dim) % 64)
-        return bad("q/k/v widths must tile by 128");
-    if (k.intermediate % 64 || (2 * k.intermediate) % 128) return bad("intermediate must be a multiple of 64");
+    if (k.hidden % 256 || k.hidden > 4096) return bad("hidden must be a multiple of 256, at most 4096");
+    if ((k.n_q_heads * k.head_dim) % 256 || ((k.n_q_heads + 2 * k.n_kv_heads) * k.head_dim) % 128)
+        return bad("q/k/v widths must tile by 128 and the attention width by 256");
+    if (k.intermediate % 256) return bad("intermediate must be a multiple of 256");
     if (k.vocab % 128) return bad("vocab must be a multiple of 128");
     if (k.lora_rank < 1 || k.lora_rank > 32) return bad("lora_rank must be in [1, 32]");
     if (k.page_size != PAGE) return bad("page_size must be 16");
     if (k.block_D < 1 || k.block_D > 64) return bad("block_D must be in [1, 64]");
     if (k.max_batch < 1 || k.max_batch > 64) return bad("max_batch must be in [1, 64]");
-    if (k.max_batch * (k.block_D + 1) > 1024) return bad("max_batch * (block_D + 1) must be <= 1024");
+    if (k.max_batch * (k.block_D + 1) > 256) return bad("max_batch * (block_D + 1) must be <= 256");
     if (k.max_seq_len < 2 || k.max_seq_len > (1 << 20)) return bad("max_seq_len out of range");
     if (!(k.rms_eps > 0.f) || !(k.rope_theta > 0.f)) return bad("rms_eps and rope_theta must be positive");
     return true;
+}
+
+int lin_K(const pbd_config &k, int lin) {
+    return lin == 1 ? k.n_q_heads * k.head_dim : (lin == 3 ? k.intermediate : k.hidden);
+}
+int lin_main(const pbd_config &k, int lin) {
+    return lin == 0 ? (k.n_q_heads + 2 * k.n_kv_heads) * k.head_dim
+                    : (lin == 2 ? 2 * k.intermediate : k.hidden);
+}
+int lin_lora(const pbd_config &k, int lin) {
+    return k.lora_rank * (lin == 0 ? 3 : (lin == 2 ? 2 : 1));
 }
 
 // Carves the workspace; with base == nullptr it only measures.  Returns total bytes.
@@ -168,7 +189,7 @@ size_t layout(pbd_ctx *c, void *base) {
     const int nl = k.n_layers, H = k.hidden, d = k.head_dim, Hq = k.n_q_heads, Hkv = k.n_kv_heads;
     const int I = k.intermediate, V = k.vocab, r = k.lora_rank, D = k.block_D;
     c->D = D;
-    c->rows_alloc = std::max(((k.max_batch * (D + 1) + 255) / 256) * 256, PREFILL_ROWS);
+    c->rows_alloc = ((std::max(k.max_batch * (D + 1), PREFILL_ROWS) + 31) / 32) * 32;
     c->ro_alloc = k.max_batch * (D + 1);
     c->out_cap = k.max_seq_len;
     // a truncated last round can leave L up to D past the budget, and every later pass still
@@ -178,13 +199,18 @@ size_t layout(pbd_ctx *c, void *base) {
     c->n_splits = (max_tokens + ATT_SPLIT - 1) / ATT_SPLIT;
     c->pages_per_seq = (max_tokens + PAGE - 1) / PAGE;
     c->n_pages = k.max_batch * c->pages_per_seq;
+    if (c->grid <= 0) c->grid = 160;  // measuring only; pbd_create uses the device's SM count
     const int B = k.max_batch, RA = c->rows_alloc;
+    mk_counter_layout(c->dm, B, &c->cl);
+    size_t lin_items = 0;
+    for (int lin = 0; lin < 4; ++lin) lin_items += (size_t)(lin_main(k, lin) / TILE_ROWS + 1) * (lin_K(k, lin) / 256);
+    c->items_cap = (size_t)RA + (size_t)nl * (lin_items + (size_t)B * Hkv * c->n_splits) + (size_t)c->ro_alloc;
 
     Bump bp(base);
-    // device state and small buffers
     c->status = (int *)bp.take(64);
     c->s.all_done = c->status + 1;
     c->s.round = c->status + 2;
+    c->cnt = (int *)bp.take(sizeof(int) * (size_t)(c->cl.total + 1));
     c->s.stats = (long long *)bp.take(3 * sizeof(long long));
     c->s.L = (int *)bp.take(sizeof(int) * B);
     c->s.pending = (int *)bp.take(sizeof(int) * B);
@@ -197,34 +223,29 @@ size_t layout(pbd_ctx *c, void *base) {
     c->first_id = (int *)bp.take(sizeof(int) * 4);
     c->page_table = (int *)bp.take(sizeof(int) * (size_t)B * c->pages_per_seq);
     c->rope_cs = (float2 *)bp.take(sizeof(float2) * (size_t)c->rope_rows * (d / 2));
+    for (int p = 0; p < N_PK; ++p) {
+        c->sched[p].items = (MKItem *)bp.take(sizeof(MKItem) * c->items_cap);
+        c->sched[p].off = (int *)bp.take(sizeof(int) * (size_t)(c->grid + 1));
+        c->sched[p].nsplit = (int *)bp.take(sizeof(int) * B);
+    }
 
     // weights
-    auto tiled = [&](int n_main, int lora_rows, int K) {
-        TiledWeight w;
-        w.n_main = n_main;
-        w.lora_rows = lora_rows;
-        w.K = K;
-        const int row_tiles = n_main / TILE_ROWS + (lora_rows > 0 ? 1 : 0);
-        w.tiles = bp.take((size_t)row_tiles * (K / KT) * TILE_BYTES);
-        return w;
-    };
-    c->w_qkv.assign(nl, TiledWeight());
-    c->w_o.assign(nl, TiledWeight());
-    c->w_gu.assign(nl, TiledWeight());
-    c->w_down.assign(nl, TiledWeight());
-    const int n_qkv = (Hq + 2 * Hkv) * d;
-    for (int l = 0; l < nl; ++l) {
-        c->w_qkv[l] = tiled(n_qkv, 3 * r, H);
-        c->w_o[l] = tiled(H, r, Hq * d);
-        c->w_gu[l] = tiled(2 * I, 2 * r, H);
-        c->w_down[l] = tiled(H, r, I);
+    for (int lin = 0; lin < 4; ++lin) {
+        c->w[lin].assign(nl, TiledWeight());
+        for (int l = 0; l < nl; ++l) {
+            TiledWeight &w = c->w[lin][l];
+            w.n_main = lin_main(k, lin);
+            w.lora_rows = lin_lora(k, lin);
+            w.K = lin_K(k, lin);
+            w.tiles = bp.take((size_t)(w.n_main / TILE_ROWS + 1) * (w.K / KT) * TILE_BYTES);
+        }
     }
-    c->w_lm = tiled(V, 0, H);
+    c->w_lm.n_main = V;
+    c->w_lm.lora_rows = 0;
+    c->w_lm.K = H;
+    c->w_lm.tiles = bp.take((size_t)(V / TILE_ROWS) * (H / KT) * TILE_BYTES);
     const size_t e2 = 2;
-    c->lb_qkv = bp.take(e2 * nl * n_qkv * r);
-    c->lb_o = bp.take(e2 * nl * H * r);
-    c->lb_gu = bp.take(e2 * nl * 2 * I * r);
-    c->lb_down = bp.take(e2 * nl * H * r);
+    for (int lin = 0; lin < 4; ++lin) c->lb[lin] = bp.take(e2 * nl * (size_t)lin_main(k, lin) * r);
     c->attn_norm = bp.take(e2 * nl * H);
     c->mlp_norm = bp.take(e2 * nl * H);
     c->q_norm = bp.take(e2 * nl * d);
@@ -240,20 +261,18 @@ size_t layout(pbd_ctx *c, void *base) {
     c->kv.pages_per_seq = c->pages_per_seq;
     c->kv.n_pages = c->n_pages;
 
-    // activations and scratch
+    // activations and pass scratch
     c->h = bp.take(e2 * RA * H);
-    c->x = bp.take(e2 * RA * H);
     c->q = bp.take(e2 * RA * Hq * d);
     c->attn = bp.take(e2 * RA * Hq * d);
     c->act = bp.take(e2 * RA * I);
     c->x_ro = bp.take(e2 * c->ro_alloc * H);
-    size_t pf = 0;
-    pf = std::max(pf, (size_t)k_splits_for(H) * RA * (n_qkv + 3 * r));
-    pf = std::max(pf, (size_t)k_splits_for(Hq * d) * RA * (H + r));
-    pf = std::max(pf, (size_t)k_splits_for(H) * RA * (2 * I + 2 * r));
-    pf = std::max(pf, (size_t)k_splits_for(I) * RA * (H + r));
-    c->part_floats = pf;
-    c->part = (float *)bp.take(sizeof(float) * pf);
+    c->ss = (float *)bp.take(sizeof(float) * RA * (H / TILE_ROWS));
+    for (int lin = 0; lin < 4; ++lin) {
+        c->part[lin] = (float *)bp.take(sizeof(float) * (size_t)(lin_K(k, lin) / 256) * RA *
+                                        (lin_main(k, lin) + lin_lora(k, lin)));
+        c->red_lora[lin] = (float *)bp.take(sizeof(float) * (size_t)RA * lin_lora(k, lin));
+    }
     c->o_part = (float *)bp.take(sizeof(float) * (size_t)RA * Hq * c->n_splits * d);
     c->ml_part = (float2 *)bp.take(sizeof(float2) * (size_t)RA * Hq * c->n_splits);
     c->tile_max = (float *)bp.take(sizeof(float) * (size_t)(V / TILE_ROWS) * c->ro_alloc);
@@ -261,37 +280,18 @@ size_t layout(pbd_ctx *c, void *base) {
     return bp.off + ALIGN;
 }
 
-Partials partials_for(pbd_ctx *c, const TiledWeight &w) {
-    Partials p;
-    p.p = c->part;
-    p.k_splits = k_splits_for(w.K);
-    p.rows_alloc = c->rows_alloc;
-    p.n_total = w.n_main + w.lora_rows;
-    return p;
-}
-
 pbd_status make_maps(pbd_ctx *c) {
-    const pbd_config &k = c->cfg;
-    struct {
-        void *p;
-        int rows, cols;
-    } bufs[N_AB] = {{c->x, c->rows_alloc, k.hidden},
-                    {c->attn, c->rows_alloc, k.n_q_heads * k.head_dim},
-                    {c->act, c->rows_alloc, k.intermediate},
-                    {c->x_ro, c->ro_alloc, k.hidden}};
-    for (int a = 0; a < N_AB; ++a)
-        for (int i = 0; i < N_BN; ++i)
-            if (!encode_bf16_map(&c->maps[a][i], bufs[a].p, bufs[a].rows, bufs[a].cols, BN_CHOICES[i]))
-                return fail(c, PBD_ERR_CUDA, "tensor map encode failed (buffer %d, box rows %d)", a, BN_CHOICES[i]);
+    for (int i = 0; i < N_BN; ++i)
+        if (!encode_bf16_map(&c->maps[i], c->x_ro, c->ro_alloc, c->cfg.hidden, BN_CHOICES[i]))
+            return fail(c, PBD_ERR_CUDA, "tensor map encode failed (box rows %d)", BN_CHOICES[i]);
     return PBD_OK;
 }
 
-// Copy rows of a layer-stacked source into a tiled weight at a row offset.
 pbd_status repack(pbd_ctx *c, const void *src, size_t layer_elems, int l, int rows, int K, const TiledWeight &w,
-                  int row0) {
+                  int row0, int group = 0, int stride = 0) {
     if (!src) return fail(c, PBD_ERR_INVALID_ARG, "null weight pointer");
     const void *p = static_cast<const uint8_t *>(src) + 2 * layer_elems * l;
-    CK(launch_repack_tiled(p, rows, K, const_cast<void *>(w.tiles), row0, c->st));
+    CK(launch_repack_tiled_map(p, rows, K, const_cast<void *>(w.tiles), row0, group ? group : rows, stride, c->st));
     return PBD_OK;
 }
 
@@ -301,42 +301,35 @@ pbd_status copy_dev(pbd_ctx *c, void *dst, const void *src, size_t bytes) {
     return PBD_OK;
 }
 
-#define TRY(expr)                             \
-    do {                                      \
-        pbd_status s_ = (expr);               \
-        if (s_ != PBD_OK) return s_;          \
-    } while (0)
-
 pbd_status load_weights(pbd_ctx *c, const pbd_base_weights *bw, const pbd_adapter_weights *aw) {
     const pbd_config &k = c->cfg;
     const int nl = k.n_layers, H = k.hidden, d = k.head_dim, Hq = k.n_q_heads, Hkv = k.n_kv_heads;
     const int I = k.intermediate, r = k.lora_rank;
     const int qw = Hq * d, kvw = Hkv * d, n_qkv = qw + 2 * kvw;
-    // zero the tile storage first so the padding rows of the adapter tiles are defined
-    for (int l = 0; l < nl; ++l) {
-        const TiledWeight *ws[4] = {&c->w_qkv[l], &c->w_o[l], &c->w_gu[l], &c->w_down[l]};
-        for (const TiledWeight *w : ws) {
-            const int rt = w->n_main / TILE_ROWS + (w->lora_rows > 0 ? 1 : 0);
-            CK(cudaMemsetAsync(const_cast<void *>(w->tiles), 0, (size_t)rt * (w->K / KT) * TILE_BYTES, c->st));
+    for (int lin = 0; lin < 4; ++lin)
+        for (int l = 0; l < nl; ++l) {
+            const TiledWeight &w = c->w[lin][l];
+            CK(cudaMemsetAsync(const_cast<void *>(w.tiles), 0,
+                               (size_t)(w.n_main / TILE_ROWS + 1) * (w.K / KT) * TILE_BYTES, c->st));
         }
-    }
     const size_t e2 = 2;
     for (int l = 0; l < nl; ++l) {
-        // fused q|k|v rows, then the adapter's A_q, A_k, A_v rows
-        TRY(repack(c, bw->w[0], (size_t)qw * H, l, qw, H, c->w_qkv[l], 0));
-        TRY(repack(c, bw->w[1], (size_t)kvw * H, l, kvw, H, c->w_qkv[l], qw));
-        TRY(repack(c, bw->w[2], (size_t)kvw * H, l, kvw, H, c->w_qkv[l], qw + kvw));
-        for (int t = 0; t < 3; ++t) TRY(repack(c, aw->lora_a[t], (size_t)r * H, l, r, H, c->w_qkv[l], n_qkv + t * r));
-        TRY(repack(c, bw->w[3], (size_t)H * qw, l, H, qw, c->w_o[l], 0));
-        TRY(repack(c, aw->lora_a[3], (size_t)r * qw, l, r, qw, c->w_o[l], H));
-        TRY(repack(c, bw->w[4], (size_t)I * H, l, I, H, c->w_gu[l], 0));
-        TRY(repack(c, bw->w[5], (size_t)I * H, l, I, H, c->w_gu[l], I));
-        TRY(repack(c, aw->lora_a[4], (size_t)r * H, l, r, H, c->w_gu[l], 2 * I));
-        TRY(repack(c, aw->lora_a[5], (size_t)r * H, l, r, H, c->w_gu[l], 2 * I + r));
-        TRY(repack(c, bw->w[6], (size_t)H * I, l, H, I, c->w_down[l], 0));
-        TRY(repack(c, aw->lora_a[6], (size_t)r * I, l, r, I, c->w_down[l], H));
-        // adapter B matrices, fused in the same output order as the main rows
-        uint8_t *lq = static_cast<uint8_t *>(c->lb_qkv) + e2 * (size_t)l * n_qkv * r;
+        // q|k|v rows, then the adapter's A_q, A_k, A_v rows in the extra tile
+        TRY(repack(c, bw->w[0], (size_t)qw * H, l, qw, H, c->w[0][l], 0));
+        TRY(repack(c, bw->w[1], (size_t)kvw * H, l, kvw, H, c->w[0][l], qw));
+        TRY(repack(c, bw->w[2], (size_t)kvw * H, l, kvw, H, c->w[0][l], qw + kvw));
+        for (int t = 0; t < 3; ++t) TRY(repack(c, aw->lora_a[t], (size_t)r * H, l, r, H, c->w[0][l], n_qkv + t * r));
+        TRY(repack(c, bw->w[3], (size_t)H * qw, l, H, qw, c->w[1][l], 0));
+        TRY(repack(c, aw->lora_a[3], (size_t)r * qw, l, r, qw, c->w[1][l], H));
+        // gate and up interleaved in 64-row blocks: tile t = [gate 64t..64t+63 | up 64t..64t+63]
+        TRY(repack(c, bw->w[4], (size_t)I * H, l, I, H, c->w[2][l], 0, 64, 128));
+        TRY(repack(c, bw->w[5], (size_t)I * H, l, I, H, c->w[2][l], 64, 64, 128));
+        TRY(repack(c, aw->lora_a[4], (size_t)r * H, l, r, H, c->w[2][l], 2 * I));
+        TRY(repack(c, aw->lora_a[5], (size_t)r * H, l, r, H, c->w[2][l], 2 * I + r));
+        TRY(repack(c, bw->w[6], (size_t)H * I, l, H, I, c->w[3][l], 0));
+        TRY(repack(c, aw->lora_a[6], (size_t)r * I, l, r, I, c->w[3][l], H));
+        // adapter B matrices, fused per layer: q|k|v rows, o rows, gate rows then up rows, down rows
+        uint8_t *lq = static_cast<uint8_t *>(c->lb[0]) + e2 * (size_t)l * n_qkv * r;
         const int outs[3] = {qw, kvw, kvw};
         size_t off = 0;
         for (int t = 0; t < 3; ++t) {
@@ -345,13 +338,13 @@ pbd_status load_weights(pbd_ctx *c, const pbd_base_weights *bw, const pbd_adapte
                          e2 * (size_t)outs[t] * r));
             off += e2 * (size_t)outs[t] * r;
         }
-        TRY(copy_dev(c, static_cast<uint8_t *>(c->lb_o) + e2 * (size_t)l * H * r,
+        TRY(copy_dev(c, static_cast<uint8_t *>(c->lb[1]) + e2 * (size_t)l * H * r,
                      static_cast<const uint8_t *>(aw->lora_b[3]) + e2 * (size_t)l * H * r, e2 * (size_t)H * r));
-        uint8_t *lg = static_cast<uint8_t *>(c->lb_gu) + e2 * (size_t)l * 2 * I * r;
+        uint8_t *lg = static_cast<uint8_t *>(c->lb[2]) + e2 * (size_t)l * 2 * I * r;
         TRY(copy_dev(c, lg, static_cast<const uint8_t *>(aw->lora_b[4]) + e2 * (size_t)l * I * r, e2 * (size_t)I * r));
         TRY(copy_dev(c, lg + e2 * (size_t)I * r, static_cast<const uint8_t *>(aw->lora_b[5]) + e2 * (size_t)l * I * r,
                      e2 * (size_t)I * r));
-        TRY(copy_dev(c, static_cast<uint8_t *>(c->lb_down) + e2 * (size_t)l * H * r,
+        TRY(copy_dev(c, static_cast<uint8_t *>(c->lb[3]) + e2 * (size_t)l * H * r,
                      static_cast<const uint8_t *>(aw->lora_b[6]) + e2 * (size_t)l * H * r, e2 * (size_t)H * r));
     }
     TRY(repack(c, bw->embed, 0, 0, k.vocab, H, c->w_lm, 0));
@@ -378,47 +371,6 @@ pbd_status build_rope(pbd_ctx *c) {
     return PBD_OK;
 }
 
-// One forward pass of nb sequences x R rows through all layers and the lm_head.
-pbd_status run_pass(pbd_ctx *c, const PassDesc &pd, int *ids_out, float *logits) {
-    const Dims &dm = c->dm;
-    const int nl = dm.nl;
-    const int bn = pick_bn(pd.M), bi = bn_index(bn);
-    cudaStream_t st = c->st;
-    CK(launch_embed_norm(dm, pd, c->ids, c->w_lm.tiles, c->mask_embed, c->attn_norm, c->h, c->x, c->status, st));
-    const size_t e2 = 2;
-    const int n_qkv = (dm.Hq + 2 * dm.Hkv) * dm.d;
-    for (int l = 0; l < nl; ++l) {
-        const Partials pq = partials_for(c, c->w_qkv[l]);
-        CK(launch_linear_partials(&c->maps[AB_X][bi], bn, c->w_qkv[l], pd.adapter, pd.M, pq, c->status, st));
-        CK(launch_qkv_finalize(dm, pd, l, pq, static_cast<uint8_t *>(c->lb_qkv) + e2 * (size_t)l * n_qkv * dm.r,
-                               c->q_norm, c->k_norm, c->rope_cs, c->rope_rows, c->s.L, c->kv, c->q, c->status, st));
-        CK(launch_attention(dm, pd, l, c->q, c->kv, c->s.L, c->n_splits, c->o_part, c->ml_part, st));
-        CK(launch_attn_combine(dm, pd, c->s.L, c->n_splits, c->o_part, c->ml_part, c->attn, st));
-        const Partials po = partials_for(c, c->w_o[l]);
-        CK(launch_linear_partials(&c->maps[AB_ATTN][bi], bn, c->w_o[l], pd.adapter, pd.M, po, c->status, st));
-        CK(launch_residual_norm(dm, pd, po, dm.H, static_cast<uint8_t *>(c->lb_o) + e2 * (size_t)l * dm.H * dm.r,
-                                static_cast<uint8_t *>(c->mlp_norm) + e2 * (size_t)l * dm.H, c->h, c->x, nullptr, st));
-        const Partials pg = partials_for(c, c->w_gu[l]);
-        CK(launch_linear_partials(&c->maps[AB_X][bi], bn, c->w_gu[l], pd.adapter, pd.M, pg, c->status, st));
-        CK(launch_act(dm, pd, pg, static_cast<uint8_t *>(c->lb_gu) + e2 * (size_t)l * 2 * dm.I * dm.r, c->act, st));
-        const Partials pdn = partials_for(c, c->w_down[l]);
-        CK(launch_linear_partials(&c->maps[AB_ACT][bi], bn, c->w_down[l], pd.adapter, pd.M, pdn, c->status, st));
-        const void *gain = (l + 1 < nl) ? static_cast<const void *>(static_cast<uint8_t *>(c->attn_norm) +
-                                                                    e2 * (size_t)(l + 1) * dm.H)
-                                        : c->final_norm;
-        CK(launch_residual_norm(dm, pd, pdn, dm.H, static_cast<uint8_t *>(c->lb_down) + e2 * (size_t)l * dm.H * dm.r,
-                                gain, c->h, c->x, (l + 1 == nl) ? c->x_ro : nullptr, st));
-    }
-    const int n_ro = pd.nb * pd.ro_count;
-    if (n_ro > 0) {
-        const int bro = pick_bn(n_ro);
-        CK(launch_lm_head(&c->maps[AB_XRO][bn_index(bro)], bro, c->w_lm, n_ro, c->tile_max, c->tile_arg, logits,
-                          c->status, st));
-        CK(launch_argmax_reduce(c->tile_max, c->tile_arg, dm.V / TILE_ROWS, n_ro, ids_out, st));
-    }
-    return PBD_OK;
-}
-
 PassDesc block_pass(pbd_ctx *c, int kind) {
     PassDesc pd;
     pd.b0 = 0;
@@ -432,16 +384,107 @@ PassDesc block_pass(pbd_ctx *c, int kind) {
     return pd;
 }
 
+// Builds a pass schedule on the host and uploads it (synchronously) into slot `kind`.
+pbd_status upload_schedule(pbd_ctx *c, int kind, const PassDesc &pd, const std::vector<int> &nsplit) {
+    std::vector<MKItem> items;
+    std::vector<int> off;
+    mk_build_schedule(c->dm, pd, nsplit, c->grid, &items, &off);
+    if (items.size() > c->items_cap)
+        return fail(c, PBD_ERR_CAPACITY, "pass schedule of %zu items exceeds %zu", items.size(), c->items_cap);
+    Sched &s = c->sched[kind];
+    CK(cudaMemcpy(s.items, items.data(), items.size() * sizeof(MKItem), cudaMemcpyHostToDevice));
+    CK(cudaMemcpy(s.off, off.data(), off.size() * sizeof(int), cudaMemcpyHostToDevice));
+    CK(cudaMemcpy(s.nsplit, nsplit.data(), nsplit.size() * sizeof(int), cudaMemcpyHostToDevice));
+    s.valid = true;
+    return PBD_OK;
+}
+
+MKLaunch make_launch(pbd_ctx *c, const PassDesc &pd, int kind) {
+    MKLaunch L;
+    const pbd_config &k = c->cfg;
+    L.dm = c->dm;
+    L.pd = pd;
+    L.grid = c->grid;
+    L.items = c->sched[kind].items;
+    L.cta_off = c->sched[kind].off;
+    L.nsplit = c->sched[kind].nsplit;
+    L.cnt = c->cnt + 1;
+    L.cl = c->cl;
+    for (int lin = 0; lin < 4; ++lin) {
+        const TiledWeight &w0 = c->w[lin][0];
+        L.wt[lin] = w0.tiles;
+        L.wt_stride[lin] = k.n_layers > 1 ? (size_t)(static_cast<const uint8_t *>(c->w[lin][1].tiles) -
+                                                     static_cast<const uint8_t *>(w0.tiles))
+                                          : 0;
+        L.n_main[lin] = w0.n_main;
+        L.lora_rows[lin] = w0.lora_rows;
+        L.K[lin] = w0.K;
+        L.lora_b[lin] = c->lb[lin];
+        L.lb_stride[lin] = (size_t)w0.n_main * k.lora_rank;
+        L.part[lin] = c->part[lin];
+        L.red_lora[lin] = c->red_lora[lin];
+    }
+    L.attn_norm = c->attn_norm;
+    L.mlp_norm = c->mlp_norm;
+    L.q_norm = c->q_norm;
+    L.k_norm = c->k_norm;
+    L.final_norm = c->final_norm;
+    L.mask_embed = c->mask_embed;
+    L.embed_tiled = c->w_lm.tiles;
+    L.rope_cs = c->rope_cs;
+    L.rope_rows = c->rope_rows;
+    L.kv = c->kv;
+    L.Lbuf = c->s.L;
+    L.ids = c->ids;
+    L.part_rows = c->rows_alloc;
+    L.h = c->h;
+    L.q = c->q;
+    L.attn = c->attn;
+    L.act = c->act;
+    L.x_ro = c->x_ro;
+    L.ss = c->ss;
+    L.o_part = c->o_part;
+    L.ml_part = c->ml_part;
+    L.att_splits_alloc = c->n_splits;
+    L.status = c->status;
+    L.abort = c->cnt;
+    return L;
+}
+
+// Zero the pass counters and launch the persistent kernel for all decoder layers.
+pbd_status enqueue_pass_kernel(pbd_ctx *c, const PassDesc &pd, int kind) {
+    CK(cudaMemsetAsync(c->cnt, 0, sizeof(int) * (size_t)(c->cl.total + 1), c->st));
+    CK(launch_pass_kernel(make_launch(c, pd, kind), c->st));
+    return PBD_OK;
+}
+
+// lm_head + argmax over the read-out rows written by the pass kernel
+pbd_status enqueue_readout(pbd_ctx *c, const PassDesc &pd, int *ids_out, float *logits) {
+    const int n_ro = pd.nb * pd.ro_count;
+    if (n_ro <= 0) return PBD_OK;
+    const int bro = pick_bn(n_ro);
+    CK(launch_lm_head(&c->maps[bn_index(bro)], bro, c->w_lm, n_ro, c->tile_max, c->tile_arg, logits, c->status,
+                      c->st));
+    CK(launch_argmax_reduce(c->tile_max, c->tile_arg, c->cfg.vocab / TILE_ROWS, n_ro, ids_out, c->st));
+    return PBD_OK;
+}
+
+pbd_status run_pass(pbd_ctx *c, const PassDesc &pd, int kind, int *ids_out, float *logits) {
+    if (!c->sched[kind].valid) return fail(c, PBD_ERR_STATE, "no schedule for pass kind %d", kind);
+    TRY(enqueue_pass_kernel(c, pd, kind));
+    return enqueue_readout(c, pd, ids_out, logits);
+}
+
 pbd_status enqueue_draft(pbd_ctx *c, float *logits) {
     const PassDesc pd = block_pass(c, PK_DRAFT);
     CK(launch_build_ids(pd, 0, c->s.pending, nullptr, c->D, c->ids, c->st));
-    return run_pass(c, pd, c->draft_ids, logits);
+    return run_pass(c, pd, PK_DRAFT, c->draft_ids, logits);
 }
 
 pbd_status enqueue_verify(pbd_ctx *c, const int *drafts, float *logits) {
     const PassDesc pd = block_pass(c, PK_VERIFY);
     CK(launch_build_ids(pd, 1, c->s.pending, drafts, c->D, c->ids, c->st));
-    return run_pass(c, pd, c->verify_ids, logits);
+    return run_pass(c, pd, PK_VERIFY, c->verify_ids, logits);
 }
 
 pbd_status enqueue_accept(pbd_ctx *c, const int *forced, int *accepted) {
@@ -450,10 +493,13 @@ pbd_status enqueue_accept(pbd_ctx *c, const int *forced, int *accepted) {
     return PBD_OK;
 }
 
-pbd_status enqueue_decode(pbd_ctx *c, float *logits) {
+pbd_status enqueue_decode_pass(pbd_ctx *c, float *logits) {
     const PassDesc pd = block_pass(c, PK_DECODE);
     CK(launch_build_ids(pd, 2, c->s.pending, nullptr, 0, c->ids, c->st));
-    TRY(run_pass(c, pd, c->verify_ids, logits));
+    return run_pass(c, pd, PK_DECODE, c->verify_ids, logits);
+}
+
+pbd_status enqueue_decode_commit(pbd_ctx *c) {
     CK(launch_accept_commit(c->s, c->batch, 0, c->draft_ids, c->verify_ids, nullptr, c->batch, c->max_new, c->out_cap,
                             nullptr, c->st));
     return PBD_OK;
@@ -463,8 +509,36 @@ pbd_status check_device(pbd_ctx *c) {
     CK(cudaStreamSynchronize(c->st));
     int code = 0;
     CK(cudaMemcpy(&code, c->status, sizeof(int), cudaMemcpyDeviceToHost));
-    if (code != 0) return fail(c, PBD_ERR_DEVICE, "device status %d latched by a kernel", code);
+    if (code != 0) {
+        CK(cudaMemset(c->status, 0, sizeof(int)));  // reported once; the context stays usable
+        return fail(c, PBD_ERR_DEVICE, "device status %d latched by a kernel", code);
+    }
     return PBD_OK;
+}
+
+// attention split items per sequence over the whole generation (positions up to P + max_new + 2(D+1))
+std::vector<int> decode_splits(pbd_ctx *c) {
+    std::vector<int> ns(c->batch);
+    for (int b = 0; b < c->batch; ++b) {
+        const int tmax = std::min(c->prompt_lens[b] + c->max_new + 2 * (c->D + 1), c->pages_per_seq * PAGE);
+        ns[b] = std::min(c->n_splits, (tmax + ATT_SPLIT - 1) / ATT_SPLIT);
+    }
+    return ns;
+}
+
+double pass_bytes(pbd_ctx *c, int kind, const std::vector<int> &Ls) {
+    const pbd_config &k = c->cfg;
+    double w = 0, lora = 0;
+    for (int lin = 0; lin < 4; ++lin) {
+        w += 2.0 * lin_main(k, lin) * lin_K(k, lin);
+        lora += 2.0 * k.lora_rank * (lin_K(k, lin) + lin_main(k, lin));
+    }
+    double bytes = k.n_layers * (w + (kind == PK_DRAFT ? lora : 0.0));
+    bytes += 2.0 * (2.0 * k.n_layers * k.hidden + 2.0 * k.n_layers * k.head_dim);  // norm gains
+    const double kv_tok = 2.0 * 2.0 * k.n_layers * k.n_kv_heads * k.head_dim;
+    const int rows = kind == PK_DECODE ? 1 : c->D + 1;
+    for (int L : Ls) bytes += kv_tok * (L + rows);
+    return bytes;
 }
 
 }  // namespace
@@ -476,6 +550,9 @@ size_t pbd_workspace_bytes(const pbd_config *cfg) {
     if (!valid_config(cfg, &why)) return 0;
     pbd_ctx tmp;
     tmp.cfg = *cfg;
+    tmp.dm = Dims{cfg->n_layers, cfg->hidden,      cfg->n_q_heads, cfg->n_kv_heads, cfg->head_dim,
+                  cfg->intermediate, cfg->vocab, cfg->lora_rank, cfg->rms_eps,     cfg->lora_scale};
+    tmp.grid = 256;  // upper bound of SMs per device for the per-CTA schedule offsets
     return layout(&tmp, nullptr);
 }
 
@@ -491,21 +568,26 @@ pbd_status pbd_create(const pbd_config *cfg, const pbd_base_weights *base, const
         return fail(c, PBD_ERR_WORKSPACE, "workspace missing or not 256-byte aligned");
     c = new pbd_ctx();
     c->cfg = *cfg;
+    c->dm = Dims{cfg->n_layers, cfg->hidden,      cfg->n_q_heads, cfg->n_kv_heads, cfg->head_dim,
+                 cfg->intermediate, cfg->vocab, cfg->lora_rank, cfg->rms_eps,     cfg->lora_scale};
+    c->grid = 256;
     const size_t need = layout(c, nullptr);
     if (workspace_bytes < need) {
         delete c;
         return fail(nullptr, PBD_ERR_WORKSPACE, "workspace too small: %zu < %zu bytes", workspace_bytes, need);
     }
-    // align the carve base to 1024 bytes inside the workspace
+    c->grid = mk_grid_size();
+    if (c->grid <= 0 || c->grid > 256) {
+        delete c;
+        return fail(nullptr, PBD_ERR_CUDA, "cannot query the SM count");
+    }
     uint8_t *wb = static_cast<uint8_t *>(d_workspace);
     uint8_t *b1024 = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(wb) + ALIGN - 1) & ~(uintptr_t)(ALIGN - 1));
     layout(c, b1024);
     c->st = static_cast<cudaStream_t>(d_stream);
-    c->dm = Dims{cfg->n_layers, cfg->hidden,      cfg->n_q_heads, cfg->n_kv_heads, cfg->head_dim,
-                 cfg->intermediate, cfg->vocab, cfg->lora_rank, cfg->rms_eps,     cfg->lora_scale};
     pbd_status s;
     cudaError_t e;
-    if ((e = configure_linear_kernels()) != cudaSuccess || (e = configure_attention_kernels()) != cudaSuccess) {
+    if ((e = configure_linear_kernels()) != cudaSuccess) {
         s = fail(c, PBD_ERR_CUDA, "kernel configuration: %s", cudaGetErrorString(e));
         delete c;
         return s;
@@ -518,7 +600,6 @@ pbd_status pbd_create(const pbd_config *cfg, const pbd_base_weights *base, const
     if ((e = cudaMemsetAsync(c->kv.k, 0, kv_bytes, c->st)) != cudaSuccess ||
         (e = cudaMemsetAsync(c->kv.v, 0, kv_bytes, c->st)) != cudaSuccess ||
         (e = cudaMemsetAsync(c->status, 0, 64, c->st)) != cudaSuccess ||
-        (e = cudaMemsetAsync(c->part, 0, sizeof(float) * c->part_floats, c->st)) != cudaSuccess ||
         (e = cudaStreamSynchronize(c->st)) != cudaSuccess) {
         s = fail(c, PBD_ERR_CUDA, "workspace init: %s", cudaGetErrorString(e));
         delete c;
@@ -538,13 +619,16 @@ pbd_status pbd_destroy(pbd_ctx *c) {
 pbd_status pbd_prefill(pbd_ctx *c, int32_t batch, const int32_t *d_prompt_ids, const int32_t *h_prompt_lens,
                        int32_t max_new, int32_t *d_first_token) {
     if (!c) return fail(c, PBD_ERR_INVALID_ARG, "null context");
-    if (batch < 1 || batch > c->cfg.max_batch) return fail(c, PBD_ERR_CAPACITY, "batch %d outside [1, %d]", batch, c->cfg.max_batch);
+    if (batch < 1 || batch > c->cfg.max_batch)
+        return fail(c, PBD_ERR_CAPACITY, "batch %d outside [1, %d]", batch, c->cfg.max_batch);
     if (!d_prompt_ids || !h_prompt_lens) return fail(c, PBD_ERR_INVALID_ARG, "null prompt");
     if (max_new < 1) return fail(c, PBD_ERR_INVALID_ARG, "max_new must be >= 1");
     for (int b = 0; b < batch; ++b)
         if (h_prompt_lens[b] < 1 || h_prompt_lens[b] + max_new > c->cfg.max_seq_len)
             return fail(c, PBD_ERR_CAPACITY, "sequence %d: prompt %d + max_new %d exceeds max_seq_len %d", b,
                         h_prompt_lens[b], max_new, c->cfg.max_seq_len);
+    c->drop_bench_graphs(0);
+    c->drop_bench_graphs(1);
     // pages of sequence b are interleaved across the batch: page (b, j) -> j * batch + b
     std::vector<int> pt((size_t)c->cfg.max_batch * c->pages_per_seq, 0);
     for (int b = 0; b < batch; ++b)
@@ -555,8 +639,10 @@ pbd_status pbd_prefill(pbd_ctx *c, int32_t batch, const int32_t *d_prompt_ids, c
     CK(cudaMemsetAsync(c->s.done, 0, sizeof(int) * c->cfg.max_batch, c->st));
     CK(cudaMemsetAsync(c->s.all_done, 0, 2 * sizeof(int), c->st));
     CK(cudaMemsetAsync(c->s.stats, 0, 3 * sizeof(long long), c->st));
+    CK(cudaStreamSynchronize(c->st));
     c->batch = batch;
     c->max_new = max_new;
+    c->prompt_lens.assign(h_prompt_lens, h_prompt_lens + batch);
     size_t off = 0;
     for (int b = 0; b < batch; ++b) {
         const int P = h_prompt_lens[b];
@@ -572,9 +658,12 @@ pbd_status pbd_prefill(pbd_ctx *c, int32_t batch, const int32_t *d_prompt_ids, c
             pd.mask_mode = MASK_CAUSAL;
             pd.ro_first = last ? rows - 1 : 0;
             pd.ro_count = last ? 1 : 0;
+            const std::vector<int> ns(1, (c0 + rows + ATT_SPLIT - 1) / ATT_SPLIT);
+            CK(cudaStreamSynchronize(c->st));  // the schedule slot is rewritten per chunk
+            TRY(upload_schedule(c, PK_PREFILL, pd, ns));
             CK(launch_set_len(c->s.L, b, c0, c->st));
             CK(cudaMemcpyAsync(c->ids, d_prompt_ids + off + c0, sizeof(int) * rows, cudaMemcpyDeviceToDevice, c->st));
-            TRY(run_pass(c, pd, c->first_id, nullptr));
+            TRY(run_pass(c, pd, PK_PREFILL, c->first_id, nullptr));
         }
         CK(launch_prefill_finish(c->s, b, P, c->first_id, max_new, c->out_cap, c->st));
         off += P;
@@ -582,6 +671,11 @@ pbd_status pbd_prefill(pbd_ctx *c, int32_t batch, const int32_t *d_prompt_ids, c
     if (d_first_token)
         CK(cudaMemcpyAsync(d_first_token, c->s.pending, sizeof(int) * batch, cudaMemcpyDeviceToDevice, c->st));
     TRY(check_device(c));
+    // schedules of the decode passes of this generation
+    const std::vector<int> ns = decode_splits(c);
+    TRY(upload_schedule(c, PK_DRAFT, block_pass(c, PK_DRAFT), ns));
+    TRY(upload_schedule(c, PK_VERIFY, block_pass(c, PK_VERIFY), ns));
+    TRY(upload_schedule(c, PK_DECODE, block_pass(c, PK_DECODE), ns));
     c->phase = PH_READY;
     return PBD_OK;
 }
@@ -615,9 +709,7 @@ pbd_status pbd_accept_commit(pbd_ctx *c, const int32_t *d_forced_n_opt, int32_t 
     if (!c) return fail(c, PBD_ERR_INVALID_ARG, "null context");
     if (c->phase != PH_VERIFIED) return fail(c, PBD_ERR_STATE, "accept/commit needs a verify pass first");
     // a forced length for this call only: index it as round 0 of a one-row table
-    if (d_forced_n_opt) {
-        CK(cudaMemsetAsync(c->s.round, 0, sizeof(int), c->st));
-    }
+    if (d_forced_n_opt) CK(cudaMemsetAsync(c->s.round, 0, sizeof(int), c->st));
     TRY(enqueue_accept(c, d_forced_n_opt, d_accepted_n));
     c->phase = PH_READY;
     return PBD_OK;
@@ -626,7 +718,8 @@ pbd_status pbd_accept_commit(pbd_ctx *c, const int32_t *d_forced_n_opt, int32_t 
 pbd_status pbd_decode_step(pbd_ctx *c, int32_t *d_next_opt, float *d_logits_opt) {
     if (!c) return fail(c, PBD_ERR_INVALID_ARG, "null context");
     if (c->phase != PH_READY) return fail(c, PBD_ERR_STATE, "decode step needs a prefilled or committed state");
-    TRY(enqueue_decode(c, d_logits_opt));
+    TRY(enqueue_decode_pass(c, d_logits_opt));
+    TRY(enqueue_decode_commit(c));
     if (d_next_opt) CK(cudaMemcpyAsync(d_next_opt, c->verify_ids, sizeof(int) * c->batch, cudaMemcpyDeviceToDevice, c->st));
     return PBD_OK;
 }
@@ -639,7 +732,6 @@ pbd_status pbd_generate(pbd_ctx *c, int32_t batch, const int32_t *d_prompt_ids, 
     if (!d_out_tokens) return fail(c, PBD_ERR_INVALID_ARG, "null output");
     TRY(pbd_prefill(c, batch, d_prompt_ids, h_prompt_lens, max_new, nullptr));
     CK(cudaMemsetAsync(c->s.round, 0, sizeof(int), c->st));
-    // capture one round as a graph (legacy default stream cannot be captured: run eagerly there)
     cudaGraph_t g = nullptr;
     cudaGraphExec_t ge = nullptr;
     const bool use_graph = c->st != nullptr && c->st != cudaStreamLegacy;
@@ -649,7 +741,8 @@ pbd_status pbd_generate(pbd_ctx *c, int32_t batch, const int32_t *d_prompt_ids, 
             TRY(enqueue_verify(c, c->draft_ids, nullptr));
             return enqueue_accept(c, d_forced_n_seq_opt, nullptr);
         }
-        return enqueue_decode(c, nullptr);
+        TRY(enqueue_decode_pass(c, nullptr));
+        return enqueue_decode_commit(c);
     };
     if (use_graph) {
         CK(cudaStreamBeginCapture(c->st, cudaStreamCaptureModeThreadLocal));
@@ -688,7 +781,7 @@ pbd_status pbd_generate(pbd_ctx *c, int32_t batch, const int32_t *d_prompt_ids, 
             break;
         }
         if (flags[0] != 0) {
-            result = fail(c, PBD_ERR_DEVICE, "device status %d latched by a kernel", flags[0]);
+            result = check_device(c);
             break;
         }
         if (flags[1]) break;
@@ -769,17 +862,8 @@ pbd_status pbd_bench_rounds(pbd_ctx *c, int32_t mode, int32_t warmup, int32_t st
             if (ph == 1) s = enqueue_verify(c, c->draft_ids, nullptr);
             if (ph == 2) s = enqueue_accept(c, d_forced_n_seq_opt, nullptr);
         } else {
-            const PassDesc pd = block_pass(c, PK_DECODE);
-            if (ph == 1) {
-                cudaError_t e = launch_build_ids(pd, 2, c->s.pending, nullptr, 0, c->ids, c->st);
-                s = e == cudaSuccess ? run_pass(c, pd, c->verify_ids, nullptr)
-                                     : fail(c, PBD_ERR_CUDA, "build ids: %s", cudaGetErrorString(e));
-            }
-            if (ph == 2) {
-                cudaError_t e = launch_accept_commit(c->s, c->batch, 0, c->draft_ids, c->verify_ids, nullptr,
-                                                     c->batch, c->max_new, c->out_cap, nullptr, c->st);
-                if (e != cudaSuccess) s = fail(c, PBD_ERR_CUDA, "accept: %s", cudaGetErrorString(e));
-            }
+            if (ph == 1) s = enqueue_decode_pass(c, nullptr);
+            if (ph == 2) s = enqueue_decode_commit(c);
         }
         cudaError_t e = cudaStreamEndCapture(c->st, &g);
         if (s == PBD_OK && e != cudaSuccess) s = fail(c, PBD_ERR_CUDA, "capture: %s", cudaGetErrorString(e));
@@ -801,12 +885,9 @@ pbd_status pbd_bench_rounds(pbd_ctx *c, int32_t mode, int32_t warmup, int32_t st
         c->bench_forced[mode] = d_forced_n_seq_opt;
         c->bench_nodes[mode] = nodes;
     }
-    std::vector<cudaEvent_t> ev;
-    if (s == PBD_OK) {
-        ev.resize((size_t)steps * 4, nullptr);
-        for (auto &x : ev)
-            if (cudaEventCreate(&x) != cudaSuccess) s = fail(c, PBD_ERR_CUDA, "event create");
-    }
+    std::vector<cudaEvent_t> ev((size_t)steps * 4, nullptr);
+    for (auto &x : ev)
+        if (s == PBD_OK && cudaEventCreate(&x) != cudaSuccess) s = fail(c, PBD_ERR_CUDA, "event create");
     for (int i = 0; s == PBD_OK && i < warmup + steps; ++i) {
         const bool timed = i >= warmup;
         cudaEvent_t *e4 = timed ? &ev[(size_t)(i - warmup) * 4] : nullptr;
@@ -846,47 +927,41 @@ pbd_status pbd_bench_rounds(pbd_ctx *c, int32_t mode, int32_t warmup, int32_t st
     return check_device(c);
 }
 
-pbd_status pbd_time_linear(pbd_ctx *c, int32_t which, int32_t rows, int32_t adapter, int32_t iters,
-                           double *h_ms_per_launch, double *h_weight_bytes) {
+pbd_status pbd_time_pass(pbd_ctx *c, int32_t kind, int32_t iters, double *h_ms_per_launch, double *h_bytes_per_launch) {
     if (!c || !h_ms_per_launch) return fail(c, PBD_ERR_INVALID_ARG, "null argument");
-    if (which < 0 || which > 4 || iters < 1) return fail(c, PBD_ERR_INVALID_ARG, "which in [0,4], iters >= 1");
-    const int max_rows = which == 4 ? c->ro_alloc : c->rows_alloc;
-    if (rows < 1 || rows > max_rows) return fail(c, PBD_ERR_CAPACITY, "rows outside [1, %d]", max_rows);
-    const int bn = pick_bn(rows), bi = bn_index(bn);
-    const int nl = c->cfg.n_layers;
-    const int per_sweep = which == 4 ? 1 : nl;
-    auto launch = [&](int l) -> cudaError_t {
-        switch (which) {
-            case 0: return launch_linear_partials(&c->maps[AB_X][bi], bn, c->w_qkv[l], adapter, rows,
-                                                  partials_for(c, c->w_qkv[l]), c->status, c->st);
-            case 1: return launch_linear_partials(&c->maps[AB_ATTN][bi], bn, c->w_o[l], adapter, rows,
-                                                  partials_for(c, c->w_o[l]), c->status, c->st);
-            case 2: return launch_linear_partials(&c->maps[AB_X][bi], bn, c->w_gu[l], adapter, rows,
-                                                  partials_for(c, c->w_gu[l]), c->status, c->st);
-            case 3: return launch_linear_partials(&c->maps[AB_ACT][bi], bn, c->w_down[l], adapter, rows,
-                                                  partials_for(c, c->w_down[l]), c->status, c->st);
-            default: return launch_lm_head(&c->maps[AB_XRO][bi], bn, c->w_lm, rows, c->tile_max, c->tile_arg,
-                                           nullptr, c->status, c->st);
+    if (kind < 0 || kind > 2 || iters < 1) return fail(c, PBD_ERR_INVALID_ARG, "kind in [0,2], iters >= 1");
+    if (c->phase != PH_READY) return fail(c, PBD_ERR_STATE, "timing needs a prefilled or committed state");
+    const PassDesc pd = block_pass(c, kind);
+    CK(launch_build_ids(pd, kind == PK_DRAFT ? 0 : (kind == PK_VERIFY ? 1 : 2), c->s.pending, c->draft_ids, c->D,
+                        c->ids, c->st));
+    TRY(enqueue_pass_kernel(c, pd, kind));  // warm-up launch
+    std::vector<cudaEvent_t> ev((size_t)iters * 2, nullptr);
+    pbd_status s = PBD_OK;
+    for (auto &x : ev)
+        if (s == PBD_OK && cudaEventCreate(&x) != cudaSuccess) s = fail(c, PBD_ERR_CUDA, "event create");
+    for (int i = 0; s == PBD_OK && i < iters; ++i) {
+        cudaError_t e = cudaMemsetAsync(c->cnt, 0, sizeof(int) * (size_t)(c->cl.total + 1), c->st);
+        if (e == cudaSuccess) e = cudaEventRecord(ev[2 * i], c->st);
+        if (e == cudaSuccess) e = launch_pass_kernel(make_launch(c, pd, kind), c->st);
+        if (e == cudaSuccess) e = cudaEventRecord(ev[2 * i + 1], c->st);
+        if (e != cudaSuccess) s = fail(c, PBD_ERR_CUDA, "timed launch: %s", cudaGetErrorString(e));
+    }
+    if (s == PBD_OK && cudaStreamSynchronize(c->st) != cudaSuccess) s = fail(c, PBD_ERR_CUDA, "timing sync");
+    double tot = 0;
+    if (s == PBD_OK)
+        for (int i = 0; i < iters; ++i) {
+            float ms = 0.f;
+            cudaEventElapsedTime(&ms, ev[2 * i], ev[2 * i + 1]);
+            tot += ms;
         }
-    };
-    for (int l = 0; l < per_sweep; ++l) CK(launch(l));  // warm-up sweep
-    cudaEvent_t e0, e1;
-    CK(cudaEventCreate(&e0));
-    CK(cudaEventCreate(&e1));
-    CK(cudaEventRecord(e0, c->st));
-    for (int it = 0; it < iters; ++it)
-        for (int l = 0; l < per_sweep; ++l) CK(launch(l));
-    CK(cudaEventRecord(e1, c->st));
-    CK(cudaEventSynchronize(e1));
-    float ms = 0.f;
-    cudaEventElapsedTime(&ms, e0, e1);
-    cudaEventDestroy(e0);
-    cudaEventDestroy(e1);
-    *h_ms_per_launch = (double)ms / ((double)iters * per_sweep);
-    if (h_weight_bytes) {
-        const TiledWeight &w = which == 0 ? c->w_qkv[0] : which == 1 ? c->w_o[0] : which == 2 ? c->w_gu[0]
-                               : which == 3 ? c->w_down[0] : c->w_lm;
-        *h_weight_bytes = 2.0 * (double)w.K * (w.n_main + (adapter && which < 4 ? w.lora_rows : 0));
+    for (auto &x : ev)
+        if (x) cudaEventDestroy(x);
+    TRY(s);
+    *h_ms_per_launch = tot / iters;
+    if (h_bytes_per_launch) {
+        std::vector<int> Ls(c->batch);
+        CK(cudaMemcpy(Ls.data(), c->s.L, sizeof(int) * c->batch, cudaMemcpyDeviceToHost));
+        *h_bytes_per_launch = pass_bytes(c, kind, Ls);
     }
     return check_device(c);
 }

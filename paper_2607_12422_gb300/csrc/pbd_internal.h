@@ -6,11 +6,13 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <vector>
+
 namespace pbd {
 
 constexpr int PAGE = 16;           // KV page length in tokens
 constexpr int ATT_SPLIT = 128;     // key positions per attention split (position-aligned)
-constexpr int PREFILL_ROWS = 256;  // rows per prefill chunk
+constexpr int PREFILL_ROWS = 64;   // rows per prefill chunk
 constexpr int KT = 64;             // K elements per 128-byte swizzle atom row (bf16)
 constexpr int TILE_ROWS = 128;     // output features per tensor-core tile
 constexpr int TILE_BYTES = TILE_ROWS * KT * 2;  // 16 KiB per pre-tiled weight tile
@@ -57,6 +59,68 @@ struct Partials {
     int n_total;
 };
 
+// ---- persistent pass kernel (pass_kernel.cu) ----
+
+enum MKOp : uint8_t { MK_EMBED = 0, MK_LINEAR = 1, MK_ATTN = 2, MK_FINAL = 3 };
+
+// One work item of a pass.  MK_LINEAR: lin (0 q|k|v, 1 o, 2 gate|up, 3 down), a = row tile
+// (the adapter tile is the last one), b = 256-wide K slice.  MK_ATTN: a = sequence in the pass,
+// b = KV head, c = 128-key split.  MK_EMBED: a = row.  MK_FINAL: a = read-out index, b = row.
+struct __align__(16) MKItem {
+    uint8_t op, lin;
+    uint16_t layer;
+    int32_t a, b, c;
+};
+
+// Offsets of the pass's completion counters (ints, zeroed before every pass).
+struct CounterLayout {
+    int embed;      // rows embedded
+    int global;     // first per-layer counter
+    int per_layer;  // counters per layer
+    int lin[4];     // per-tile slice arrivals (+1 once reduced), per linear
+    int res_o, res_dn;  // residual tiles finished after o / down
+    int att;        // per (sequence, KV head): split items done (+1 once merged)
+    int total;
+};
+
+struct MKLaunch {
+    Dims dm;
+    PassDesc pd;
+    int grid;
+    const MKItem *items;
+    const int *cta_off;
+    const int *nsplit;
+    int *cnt;
+    CounterLayout cl;
+    const void *wt[4];
+    size_t wt_stride[4];
+    int n_main[4], lora_rows[4], K[4];
+    const void *lora_b[4];
+    size_t lb_stride[4];
+    const void *attn_norm, *mlp_norm, *q_norm, *k_norm, *final_norm, *mask_embed, *embed_tiled;
+    const float2 *rope_cs;
+    int rope_rows;
+    KVCache kv;
+    const int *Lbuf;
+    const int *ids;
+    float *part[4];
+    int part_rows;
+    float *red_lora[4];
+    void *h, *q, *attn, *act, *x_ro;
+    float *ss;
+    float *o_part;
+    float2 *ml_part;
+    int att_splits_alloc;
+    int *status, *abort;
+};
+
+int mk_grid_size();
+void mk_counter_layout(const Dims &dm, int max_nb, CounterLayout *cl);
+void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int> &nsplit, int grid,
+                       std::vector<MKItem> *out, std::vector<int> *off);
+size_t mk_union_bytes(int bn, int head_dim);
+cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st);
+
 // ---- launchers (each returns cudaGetLastError()) ----
 
 // Tensor-core linear: part[s][m][f] = sum over split s of x[m,k] * W[f,k], for f in the main
@@ -71,30 +135,6 @@ cudaError_t launch_lm_head(const CUtensorMap *x_map, int bn, const TiledWeight &
 
 cudaError_t launch_argmax_reduce(const float *tile_max, const int *tile_arg, int n_tiles, int rows, int *ids_out,
                                  cudaStream_t st);
-
-cudaError_t launch_embed_norm(const Dims &dm, const PassDesc &pd, const int *ids, const void *embed_tiled,
-                              const void *mask_embed, const void *gain, void *h, void *x, int *status,
-                              cudaStream_t st);
-
-cudaError_t launch_qkv_finalize(const Dims &dm, const PassDesc &pd, int layer, const Partials &part,
-                                const void *lora_b_qkv, const void *q_norm, const void *k_norm,
-                                const float2 *rope_cs, int rope_rows, const int *L, const KVCache &kv, void *q_out,
-                                int *status, cudaStream_t st);
-
-cudaError_t launch_attention(const Dims &dm, const PassDesc &pd, int layer, const void *q, const KVCache &kv,
-                             const int *L, int n_splits, float *o_part, float2 *ml_part, cudaStream_t st);
-
-cudaError_t launch_attn_combine(const Dims &dm, const PassDesc &pd, const int *L, int n_splits, const float *o_part,
-                                const float2 *ml_part, void *attn_out, cudaStream_t st);
-
-// h <- bf16(h + bf16(sum partials + s * u B^T)); x <- RMSNorm(h) * gain; read-out rows also to x_ro.
-cudaError_t launch_residual_norm(const Dims &dm, const PassDesc &pd, const Partials &part, int n_out,
-                                 const void *lora_b, const void *gain, void *h, void *x, void *x_ro,
-                                 cudaStream_t st);
-
-// act <- bf16(silu(gate) * up) from the fused gate|up partials (+ adapter delta)
-cudaError_t launch_act(const Dims &dm, const PassDesc &pd, const Partials &part, const void *lora_b_gu, void *act,
-                       cudaStream_t st);
 
 // Builds the row token ids of a pass from the device state: draft [pending, -1 x D],
 // verify [pending, drafts], decode [pending].
@@ -120,6 +160,10 @@ cudaError_t launch_accept_commit(const SeqState &s, int nb, int D, const int *dr
 // Repack rows [0, rows) of a row-major bf16 matrix [rows, K] into the tiled layout at
 // destination row offset dst_row0.
 cudaError_t launch_repack_tiled(const void *src, int rows, int K, void *dst_tiles, int dst_row0, cudaStream_t st);
+// Same, with source row i placed on tile row dst_row0 + (i / group) * stride + i % group
+// (gate and up rows interleaved in 64-row blocks inside each 128-row tile).
+cudaError_t launch_repack_tiled_map(const void *src, int rows, int K, void *dst_tiles, int dst_row0, int group,
+                                    int stride, cudaStream_t st);
 
 cudaError_t launch_read_kv(const Dims &dm, const KVCache &kv, int layer, int seq, int n, void *k_out, void *v_out,
                            cudaStream_t st);
@@ -140,6 +184,5 @@ bool encode_bf16_map(CUtensorMap *map, const void *base, int rows, int cols, int
 
 // Per-instantiation kernel attributes (dynamic shared memory), set once before any capture.
 cudaError_t configure_linear_kernels();
-cudaError_t configure_attention_kernels();
 
 }  // namespace pbd

@@ -91,9 +91,9 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     L.pbd_last_error.argtypes = [P]
     L.pbd_version.restype = C.c_char_p
     L.pbd_bench_rounds.argtypes = [P, I32, I32, I32, P, P, P]
-    L.pbd_time_linear.argtypes = [P, I32, I32, I32, I32, P, P]
+    L.pbd_time_pass.argtypes = [P, I32, I32, P, P]
     L.pbd_bench_rounds.restype = C.c_int
-    L.pbd_time_linear.restype = C.c_int
+    L.pbd_time_pass.restype = C.c_int
     L.pbd_op_linear_workspace_bytes.restype = C.c_size_t
     L.pbd_op_linear_workspace_bytes.argtypes = [I32, I32, I32, I32]
     L.pbd_op_linear.argtypes = [I32, I32, I32, I32, C.c_float, P, P, P, P, P, P, C.c_size_t, P]
@@ -344,9 +344,10 @@ class Engine:
         self._call(self.lib.pbd_bench_rounds, mode, warmup, steps, fp, ms.ctypes.data, launches.ctypes.data)
         return float(ms[0]), float(ms[1]), float(ms[2]), float(ms[3]), int(launches[0])
 
-    def pbd_time_linear(self, which: int, rows: int, adapter: int, iters: int):
-        """(ms per launch, weight bytes per launch) of the tensor-core linear kernel timed alone."""
+    def pbd_time_pass(self, kind: int, iters: int):
+        """(ms per launch, algorithmic bytes per launch) of the persistent pass kernel timed alone
+        (kind 0 draft, 1 verify, 2 plain decoding)."""
         ms = np.zeros(1, np.float64)
-        wb = np.zeros(1, np.float64)
-        self._call(self.lib.pbd_time_linear, which, rows, adapter, iters, ms.ctypes.data, wb.ctypes.data)
-        return float(ms[0]), float(wb[0])
+        nb = np.zeros(1, np.float64)
+        self._call(self.lib.pbd_time_pass, kind, iters, ms.ctypes.data, nb.ctypes.data)
+        return float(ms[0]), float(nb[0])
