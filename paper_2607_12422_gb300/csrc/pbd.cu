@@ -392,9 +392,12 @@ pbd_status upload_schedule(pbd_ctx *c, int kind, const PassDesc &pd, const std::
     if (items.size() > c->items_cap)
         return fail(c, PBD_ERR_CAPACITY, "pass schedule of %zu items exceeds %zu", items.size(), c->items_cap);
     Sched &s = c->sched[kind];
-    CK(cudaMemcpy(s.items, items.data(), items.size() * sizeof(MKItem), cudaMemcpyHostToDevice));
-    CK(cudaMemcpy(s.off, off.data(), off.size() * sizeof(int), cudaMemcpyHostToDevice));
-    CK(cudaMemcpy(s.nsplit, nsplit.data(), nsplit.size() * sizeof(int), cudaMemcpyHostToDevice));
+    // ordered on the context's stream (which may not synchronise with the legacy stream), and
+    // finished before the host vectors go away
+    CK(cudaMemcpyAsync(s.items, items.data(), items.size() * sizeof(MKItem), cudaMemcpyHostToDevice, c->st));
+    CK(cudaMemcpyAsync(s.off, off.data(), off.size() * sizeof(int), cudaMemcpyHostToDevice, c->st));
+    CK(cudaMemcpyAsync(s.nsplit, nsplit.data(), nsplit.size() * sizeof(int), cudaMemcpyHostToDevice, c->st));
+    CK(cudaStreamSynchronize(c->st));
     s.valid = true;
     return PBD_OK;
 }
