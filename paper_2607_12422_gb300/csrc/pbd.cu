@@ -513,7 +513,8 @@ pbd_status check_device(pbd_ctx *c) {
     int code = 0;
     CK(cudaMemcpy(&code, c->status, sizeof(int), cudaMemcpyDeviceToHost));
     if (code != 0) {
-        CK(cudaMemset(c->status, 0, sizeof(int)));  // reported once; the context stays usable
+        CK(cudaMemsetAsync(c->status, 0, sizeof(int), c->st));  // reported once; the context stays usable
+        CK(cudaStreamSynchronize(c->st));
         return fail(c, PBD_ERR_DEVICE, "device status %d latched by a kernel", code);
     }
     return PBD_OK;
