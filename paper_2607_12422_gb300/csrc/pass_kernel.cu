@@ -94,6 +94,7 @@ struct MKParams {
     int att_splits_alloc;
     float att_scale;           // 1/sqrt(head_dim)
     int *status, *abort;
+    unsigned long long *trace;  // optional: 4 timestamps per item (start, inputs ready, work done, end)
     // launch geometry
     int bn, nslot, ring_bytes, union_bytes;
     uint32_t tmem_cols;
@@ -154,28 +155,84 @@ __device__ __forceinline__ float tile_sumsq(const float (&v)[4]) {
     return __shfl_sync(0xffffffffu, s, 0);
 }
 
+// With one CTA per SM only six compute warps hide memory latency, so every helper below issues
+// all of its independent loads before it consumes any; sums still run in one fixed order.
+// Data written by other CTAs during the pass is read with L2-only loads (never a stale L1 line).
+constexpr int MAX_HT = 32;     // 128-feature tiles of the hidden size (H <= 4096)
+constexpr int MAX_RANK = 16;   // adapter rank (8 or 16)
+
+__device__ __forceinline__ float ldcg_bf(const bf16 *p) {
+    return __ushort_as_bfloat16(__ldcg(reinterpret_cast<const unsigned short *>(p)));
+}
+
 // 1/sqrt(mean(h^2) + eps) of row m from its per-tile sums (tiles added in order)
 __device__ __forceinline__ float row_rms(const MKParams &P, int m) {
     const int nt = P.dm.H / TILE_ROWS;
     const float *s = P.ss + (size_t)m * nt;
-    float a = s[0];
-    for (int t = 1; t < nt; ++t) a = __fadd_rn(a, s[t]);
+    float v[MAX_HT];
+#pragma unroll
+    for (int t = 0; t < MAX_HT; ++t) v[t] = t < nt ? __ldcg(s + t) : 0.f;
+    float a = v[0];
+#pragma unroll
+    for (int t = 1; t < MAX_HT; ++t)
+        if (t < nt) a = __fadd_rn(a, v[t]);
     return __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(__fdiv_rn(a, (float)P.dm.H), P.dm.eps)));
 }
 
-__device__ __forceinline__ float lora_dot_f(const float *u, const bf16 *Brow, int r) {
+// u[0..r) of row m: the bf16-rounded adapter intermediates x A^T (kept as fp32), r % 4 == 0
+__device__ __forceinline__ void load_u(const float *src, int r, float (&u)[MAX_RANK]) {
+#pragma unroll
+    for (int q = 0; q < MAX_RANK / 4; ++q) {
+        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (q * 4 < r) v = __ldcg(reinterpret_cast<const float4 *>(src) + q);
+        u[4 * q] = v.x;
+        u[4 * q + 1] = v.y;
+        u[4 * q + 2] = v.z;
+        u[4 * q + 3] = v.w;
+    }
+}
+
+// sum_j u_j * B[f, j] over j = 0..r-1 in order (B row: r bf16 values, r % 8 == 0)
+__device__ __forceinline__ float lora_dot_f(const float (&u)[MAX_RANK], const bf16 *Brow, int r) {
+    uint4 w[MAX_RANK / 8];
+#pragma unroll
+    for (int q = 0; q < MAX_RANK / 8; ++q)
+        if (q * 8 < r) w[q] = __ldg(reinterpret_cast<const uint4 *>(Brow) + q);
     float a = 0.f;
-    for (int j = 0; j < r; ++j) a = __fadd_rn(a, __fmul_rn(u[j], bf2f(Brow[j])));
+#pragma unroll
+    for (int q = 0; q < MAX_RANK / 8; ++q) {
+        if (q * 8 < r) {
+            const bf16 *e = reinterpret_cast<const bf16 *>(&w[q]);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) a = __fadd_rn(a, __fmul_rn(u[q * 8 + j], bf2f(e[j])));
+        }
+    }
     return a;
 }
 
-__device__ __forceinline__ float sum_part(const MKParams &P, int lin, int m, int f) {
+// Sums of the K-slice partials of E features of row m, slices added in order; loads go out
+// in batches of S slices (every load of a batch in flight before the first add).
+template <int E, int S>
+__device__ __forceinline__ void sum_parts(const MKParams &P, int lin, int m, const int (&f)[E], float (&out)[E]) {
     const int nt = P.n_main[lin] + P.lora_rows[lin];
-    const float *p = P.part[lin] + (size_t)m * nt + f;
+    const float *p = P.part[lin] + (size_t)m * nt;
     const size_t stride = (size_t)P.part_rows * nt;
-    float a = p[0];
-    for (int s = 1; s < P.ks[lin]; ++s) a = __fadd_rn(a, p[s * stride]);
-    return a;
+    const int ks = P.ks[lin];
+    for (int s0 = 0; s0 < ks; s0 += S) {
+        float v[E][S];
+#pragma unroll
+        for (int s = 0; s < S; ++s)
+#pragma unroll
+            for (int e = 0; e < E; ++e) v[e][s] = s0 + s < ks ? __ldcg(p + (s0 + s) * stride + f[e]) : 0.f;
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+#pragma unroll
+            for (int s = 0; s < S; ++s) {
+                if (s0 + s >= ks) break;
+                out[e] = (s0 + s == 0) ? v[e][s] : __fadd_rn(out[e], v[e][s]);
+            }
+        }
+    }
 }
 
 // element (v, k) of a matrix in the 128 x 64 swizzled tile layout
@@ -187,7 +244,7 @@ __device__ __forceinline__ const bf16 *tiled_at(const bf16 *tiles, int K, int v,
 // ------------------------------------------------------------------ work items
 
 // token / mask-embedding row -> residual h and its per-tile sums of squares
-__device__ void do_embed(const MKParams &P, int m, int cw, int lane) {
+__device__ __noinline__ void do_embed(const MKParams &P, int m, int cw, int lane) {
     int tok = P.ids[m];
     if (tok >= P.dm.V) {
         latch_error(P.status, DEV_BAD_TOKEN);
@@ -200,8 +257,9 @@ __device__ void do_embed(const MKParams &P, int m, int cw, int lane) {
         for (int e = 0; e < 4; ++e) {
             const int f = t * TILE_ROWS + lane + 32 * e;
             v[e] = tok >= 0 ? bf2f(*tiled_at(P.embed_tiled, H, tok, f)) : bf2f(P.mask_embed[f]);
-            P.h[(size_t)m * H + f] = f2bf(v[e]);
         }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) P.h[(size_t)m * H + t * TILE_ROWS + lane + 32 * e] = f2bf(v[e]);
         const float s = tile_sumsq(v);
         if (lane == 0) P.ss[(size_t)m * nt + t] = s;
     }
@@ -209,7 +267,9 @@ __device__ void do_embed(const MKParams &P, int m, int cw, int lane) {
 
 // Activation tile of one linear item in the 128-byte swizzle layout: atom j (K columns
 // 64j..64j+63 of the slice) holds row m at m*128 bytes, 16-byte chunk c at (c ^ (m & 7)) * 16.
-__device__ void build_b(const MKParams &P, int lin, int layer, int slice, uint8_t *sb, float *s_rms, int ct) {
+// Row m of the q|k|v and gate|up inputs is RMSNorm(h_m) * gain, computed here on the fly.
+__device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int slice, uint8_t *sb, float *s_rms, int ct) {
+    constexpr int U = 4;  // chunks in flight per thread
     const int M = P.pd.M;
     const int k0 = slice * KSLICE;
     const bool norm = (lin == 0 || lin == 2);
@@ -218,40 +278,55 @@ __device__ void build_b(const MKParams &P, int lin, int layer, int slice, uint8_
         bar_compute();
     }
     const bf16 *gain = lin == 0 ? P.attn_norm + (size_t)layer * P.dm.H : P.mlp_norm + (size_t)layer * P.dm.H;
+    const bf16 *src = norm ? P.h : (lin == 1 ? P.attn : P.act);
+    const int ld = norm ? P.dm.H : (lin == 1 ? P.dm.Hq * P.dm.d : P.dm.I);
     const int chunks = M * (KSLICE / 8);
-    for (int q = ct; q < chunks; q += CT) {
-        const int m = q / (KSLICE / 8), c = q % (KSLICE / 8);
-        const int atom = c >> 3, cc = c & 7;
-        uint4 val;
-        if (norm) {
-            const uint4 hv = *reinterpret_cast<const uint4 *>(P.h + (size_t)m * P.dm.H + k0 + c * 8);
-            const uint4 gv = *reinterpret_cast<const uint4 *>(gain + k0 + c * 8);
-            const bf16 *he = reinterpret_cast<const bf16 *>(&hv);
-            const bf16 *ge = reinterpret_cast<const bf16 *>(&gv);
-            bf16 *oe = reinterpret_cast<bf16 *>(&val);
-            const float rs = s_rms[m];
+    for (int q0 = ct; q0 < chunks; q0 += U * CT) {
+        uint4 xv[U], gv[U];
 #pragma unroll
-            for (int e = 0; e < 8; ++e) oe[e] = f2bf(__fmul_rn(bf2f(ge[e]), rbf(__fmul_rn(bf2f(he[e]), rs))));
-        } else {
-            const bf16 *src = lin == 1 ? P.attn + (size_t)m * (P.dm.Hq * P.dm.d) : P.act + (size_t)m * P.dm.I;
-            val = *reinterpret_cast<const uint4 *>(src + k0 + c * 8);
+        for (int u = 0; u < U; ++u) {
+            const int q = q0 + u * CT;
+            if (q < chunks) {
+                const int m = q / (KSLICE / 8), c = q % (KSLICE / 8);
+                xv[u] = __ldcg(reinterpret_cast<const uint4 *>(src + (size_t)m * ld + k0 + c * 8));
+                if (norm) gv[u] = __ldg(reinterpret_cast<const uint4 *>(gain + k0 + c * 8));
+            }
         }
-        *reinterpret_cast<uint4 *>(sb + (size_t)atom * P.bn * 128 + m * 128 + ((cc ^ (m & 7)) << 4)) = val;
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int q = q0 + u * CT;
+            if (q >= chunks) break;
+            const int m = q / (KSLICE / 8), c = q % (KSLICE / 8);
+            const int atom = c >> 3, cc = c & 7;
+            uint4 val = xv[u];
+            if (norm) {
+                const bf16 *he = reinterpret_cast<const bf16 *>(&xv[u]);
+                const bf16 *ge = reinterpret_cast<const bf16 *>(&gv[u]);
+                bf16 *oe = reinterpret_cast<bf16 *>(&val);
+                const float rs = s_rms[m];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) oe[e] = f2bf(__fmul_rn(bf2f(ge[e]), rbf(__fmul_rn(bf2f(he[e]), rs))));
+            }
+            *reinterpret_cast<uint4 *>(sb + (size_t)atom * P.bn * 128 + m * 128 + ((cc ^ (m & 7)) << 4)) = val;
+        }
     }
 }
 
 // reducer of the adapter tile: u = bf16(sum of slices), kept as fp32 values
-__device__ void reduce_lora(const MKParams &P, int lin, int ct) {
+__device__ __noinline__ void reduce_lora(const MKParams &P, int lin, int ct) {
     const int M = P.pd.M, lr = P.lora_rows[lin], n0 = P.n_main[lin];
     for (int q = ct; q < M * lr; q += CT) {
         const int m = q / lr, j = q % lr;
-        P.red_lora[lin][q] = rbf(sum_part(P, lin, m, n0 + j));
+        const int f[1] = {n0 + j};
+        float s[1];
+        sum_parts<1, 4>(P, lin, m, f, s);
+        P.red_lora[lin][q] = rbf(s[0]);
     }
 }
 
 // q|k|v tile: adapter delta, bf16, per-head RMSNorm + RoPE for q and k, store q / paged K, V
 template <int DH>
-__device__ void reduce_qkv(const MKParams &P, int layer, int tile, int cw, int lane) {
+__device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, int cw, int lane) {
     constexpr int E = DH / 32;
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r;
@@ -265,14 +340,17 @@ __device__ void reduce_qkv(const MKParams &P, int layer, int tile, int cw, int l
         const int head = kind == 0 ? fbase / DH : (kind == 1 ? (fbase - qw) / DH : (fbase - qw - kvw) / DH);
         const int b = P.pd.b0 + m / P.pd.R;
         const int pos = P.L[b] + m % P.pd.R;
-        const float *u = P.red_lora[0] + (size_t)m * P.lora_rows[0] + kind * r;
+        int f[E];
+#pragma unroll
+        for (int j = 0; j < E; ++j) f[j] = fbase + lane + 32 * j;
+        float u[MAX_RANK];
+        if (P.pd.adapter) load_u(P.red_lora[0] + (size_t)m * P.lora_rows[0] + kind * r, r, u);
         float y[E];
+        sum_parts<E, 4>(P, 0, m, f, y);
 #pragma unroll
         for (int j = 0; j < E; ++j) {
-            const int f = fbase + lane + 32 * j;
-            float acc = sum_part(P, 0, m, f);
-            if (P.pd.adapter) acc = __fadd_rn(acc, __fmul_rn(dm.lora_scale, lora_dot_f(u, lb + (size_t)f * r, r)));
-            y[j] = rbf(acc);
+            if (P.pd.adapter) y[j] = __fadd_rn(y[j], __fmul_rn(dm.lora_scale, lora_dot_f(u, lb + (size_t)f[j] * r, r)));
+            y[j] = rbf(y[j]);
         }
         if (kind < 2) {
             const bf16 *gn = (kind == 0 ? P.q_norm : P.k_norm) + (size_t)layer * DH;
@@ -318,22 +396,27 @@ __device__ void reduce_qkv(const MKParams &P, int layer, int tile, int cw, int l
 }
 
 // o or down tile: adapter delta, residual add into h, per-tile sum of squares
-__device__ void reduce_residual(const MKParams &P, int lin, int layer, int tile, int cw, int lane) {
+__device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int layer, int tile, int cw, int lane) {
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r, H = dm.H, nt = H / TILE_ROWS;
     const bf16 *lb = P.lora_b[lin] + (size_t)layer * P.lb_stride[lin];
     for (int m = cw; m < M; m += CT / 32) {
-        const float *u = P.red_lora[lin] + (size_t)m * P.lora_rows[lin];
+        int f[4];
+        float hv[4], acc[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            f[e] = tile * TILE_ROWS + lane + 32 * e;
+            hv[e] = bf2f(ldcg_bf(P.h + (size_t)m * H + f[e]));
+        }
+        float u[MAX_RANK];
+        if (P.pd.adapter) load_u(P.red_lora[lin] + (size_t)m * P.lora_rows[lin], r, u);
+        sum_parts<4, 4>(P, lin, m, f, acc);
         float v[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-            const int f = tile * TILE_ROWS + lane + 32 * e;
-            float acc = sum_part(P, lin, m, f);
-            if (P.pd.adapter) acc = __fadd_rn(acc, __fmul_rn(dm.lora_scale, lora_dot_f(u, lb + (size_t)f * r, r)));
-            const float y = rbf(acc);
-            const float hn = rbf(__fadd_rn(bf2f(P.h[(size_t)m * H + f]), y));
-            P.h[(size_t)m * H + f] = f2bf(hn);
-            v[e] = hn;
+            if (P.pd.adapter) acc[e] = __fadd_rn(acc[e], __fmul_rn(dm.lora_scale, lora_dot_f(u, lb + (size_t)f[e] * r, r)));
+            v[e] = rbf(__fadd_rn(hv[e], rbf(acc[e])));
+            P.h[(size_t)m * H + f[e]] = f2bf(v[e]);
         }
         const float s = tile_sumsq(v);
         if (lane == 0) P.ss[(size_t)m * nt + tile] = s;
@@ -341,26 +424,32 @@ __device__ void reduce_residual(const MKParams &P, int lin, int layer, int tile,
 }
 
 // gate|up tile (rows 0-63 gate features 64t.., rows 64-127 up features 64t..): SiLU(gate)*up
-__device__ void reduce_gu(const MKParams &P, int layer, int tile, int cw, int lane) {
+__device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, int cw, int lane) {
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r, I = dm.I;
     const bf16 *lb = P.lora_b[2] + (size_t)layer * P.lb_stride[2];
     for (int m = cw; m < M; m += CT / 32) {
-        const float *u = P.red_lora[2] + (size_t)m * P.lora_rows[2];
+        // partial rows: gate j = lane, lane+32 at tile rows j; up at tile rows 64 + j
+        const int f[4] = {tile * TILE_ROWS + lane, tile * TILE_ROWS + lane + 32, tile * TILE_ROWS + 64 + lane,
+                          tile * TILE_ROWS + 96 + lane};
+        float ug[MAX_RANK], uu[MAX_RANK], s[4];
+        if (P.pd.adapter) {
+            load_u(P.red_lora[2] + (size_t)m * P.lora_rows[2], r, ug);
+            load_u(P.red_lora[2] + (size_t)m * P.lora_rows[2] + r, r, uu);
+        }
+        sum_parts<4, 4>(P, 2, m, f, s);
 #pragma unroll
         for (int e = 0; e < 2; ++e) {
-            const int j = lane + 32 * e;  // 0..63
-            const int f = tile * 64 + j;  // act feature
-            float g = sum_part(P, 2, m, tile * TILE_ROWS + j);
-            float up = sum_part(P, 2, m, tile * TILE_ROWS + 64 + j);
+            const int a = tile * 64 + lane + 32 * e;  // act feature
+            float g = s[e], up = s[2 + e];
             if (P.pd.adapter) {
-                g = __fadd_rn(g, __fmul_rn(dm.lora_scale, lora_dot_f(u, lb + (size_t)f * r, r)));
-                up = __fadd_rn(up, __fmul_rn(dm.lora_scale, lora_dot_f(u + r, lb + (size_t)(I + f) * r, r)));
+                g = __fadd_rn(g, __fmul_rn(dm.lora_scale, lora_dot_f(ug, lb + (size_t)a * r, r)));
+                up = __fadd_rn(up, __fmul_rn(dm.lora_scale, lora_dot_f(uu, lb + (size_t)(I + a) * r, r)));
             }
             g = rbf(g);
             up = rbf(up);
             const float sg = __fdiv_rn(g, __fadd_rn(1.0f, expf(-g)));
-            P.act[(size_t)m * I + f] = f2bf(__fmul_rn(sg, up));
+            P.act[(size_t)m * I + a] = f2bf(__fmul_rn(sg, up));
         }
     }
 }
@@ -370,7 +459,7 @@ __device__ void reduce_gu(const MKParams &P, int layer, int tile, int cw, int la
 __device__ __forceinline__ uint32_t ldu32(const void *p) { return *reinterpret_cast<const uint32_t *>(p); }
 
 template <int DH>
-__device__ void attn_split(const MKParams &P, int layer, int bl, int g, int s, uint8_t *smem, int ct, int cw,
+__device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, int g, int s, uint8_t *smem, int ct, int cw,
                            int lane) {
     constexpr int KSTR = DH + 8, VSTR = DH + 8;
     constexpr int NT = ATT_SPLIT / 8, KS = DH / 16, DT = DH / 8;
@@ -385,25 +474,43 @@ __device__ void attn_split(const MKParams &P, int layer, int bl, int g, int s, u
     const int n_mt = (QV + 15) / 16;
     bf16 *sK = reinterpret_cast<bf16 *>(smem);
     __half *sV = reinterpret_cast<__half *>(smem + ATT_SPLIT * KSTR * 2);
+    int *s_page = reinterpret_cast<int *>(smem + ATT_SPLIT * KSTR * 2 + ATT_SPLIT * VSTR * 2);
     const size_t layer_off = (size_t)layer * P.kv.n_pages * dm.Hkv * PAGE * DH;
     const bf16 *kc = static_cast<const bf16 *>(P.kv.k), *vc = static_cast<const bf16 *>(P.kv.v);
+    // physical pages of the split (-1: beyond the keys of this pass or the reserved pages)
+    if (ct < ATT_SPLIT / PAGE) {
+        const int kp = k0 + ct * PAGE;
+        s_page[ct] = (kp < T && kp / PAGE < P.kv.pages_per_seq) ? P.kv.page_table[b * P.kv.pages_per_seq + kp / PAGE]
+                                                               : -1;
+    }
+    bar_compute();
+    // every 16-byte chunk of K and V in flight at once (async copies, zero fill past the last key)
     for (int idx = ct; idx < ATT_SPLIT * (DH / 8); idx += CT) {
         const int kk = idx / (DH / 8), c = idx % (DH / 8);
-        const int kp = k0 + kk;
-        uint4 k4 = make_uint4(0, 0, 0, 0), v4 = make_uint4(0, 0, 0, 0);
-        if (kp < T && kp / PAGE < P.kv.pages_per_seq) {
-            const int page = P.kv.page_table[b * P.kv.pages_per_seq + kp / PAGE];
-            const size_t off = layer_off + (((size_t)page * dm.Hkv + g) * PAGE + (kp % PAGE)) * DH + (size_t)c * 8;
-            k4 = *reinterpret_cast<const uint4 *>(kc + off);
-            v4 = *reinterpret_cast<const uint4 *>(vc + off);
-        }
-        *reinterpret_cast<uint4 *>(sK + kk * KSTR + c * 8) = k4;
+        const int kp = k0 + kk, page = s_page[kk / PAGE];
+        const bool ok = page >= 0 && kp < T;
+        const size_t off = ok ? layer_off + (((size_t)page * dm.Hkv + g) * PAGE + (kp % PAGE)) * DH + (size_t)c * 8 : 0;
+        const uint32_t nbytes = ok ? 16u : 0u;
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(sK + kk * KSTR + c * 8)),
+                     "l"(kc + off), "r"(nbytes)
+                     : "memory");
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(sV + kk * VSTR + c * 8)),
+                     "l"(vc + off), "r"(nbytes)
+                     : "memory");
+    }
+    asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+    bar_compute();
+    // V to fp16 in place (same size, same padded layout)
+    for (int idx = ct; idx < ATT_SPLIT * (DH / 8); idx += CT) {
+        const int kk = idx / (DH / 8), c = idx % (DH / 8);
+        uint4 *p4 = reinterpret_cast<uint4 *>(sV + kk * VSTR + c * 8);
+        const uint4 v4 = *p4;
         const bf16 *ve = reinterpret_cast<const bf16 *>(&v4);
         uint4 h4;
         uint32_t *hw = reinterpret_cast<uint32_t *>(&h4);
 #pragma unroll
         for (int e = 0; e < 4; ++e) hw[e] = pack_half2(bf2f(ve[2 * e]), bf2f(ve[2 * e + 1]));
-        *reinterpret_cast<uint4 *>(sV + kk * VSTR + c * 8) = h4;
+        *p4 = h4;
     }
     bar_compute();
     const int gq = lane >> 2, tq = lane & 3;
@@ -515,7 +622,7 @@ __device__ void attn_split(const MKParams &P, int layer, int bl, int g, int s, u
 
 // merge the splits of (row, head) in split order; splits where the row saw no key are skipped
 template <int DH>
-__device__ void attn_combine(const MKParams &P, int bl, int g, int cw, int lane) {
+__device__ __noinline__ void attn_combine(const MKParams &P, int bl, int g, int cw, int lane) {
     const Dims &dm = P.dm;
     const int R = P.pd.R, grp = dm.Hq / dm.Hkv;
     const int b = P.pd.b0 + bl;
@@ -527,23 +634,38 @@ __device__ void attn_combine(const MKParams &P, int bl, int g, int cw, int lane)
         const int i = it / grp, h = g * grp + it % grp;
         const int m = bl * R + i;
         const float2 *ml = P.ml_part + ((size_t)m * dm.Hq + h) * nsa;
+        const float *ob = P.o_part + ((size_t)m * dm.Hq + h) * nsa * DH + lane;
         float mx = -INFINITY;
-        for (int s = 0; s < nv; ++s) {
-            const float2 v = ml[s];
-            if (v.y > 0.f) mx = fmaxf(mx, v.x);
+        for (int s0 = 0; s0 < nv; s0 += 8) {
+            float2 v[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) v[u] = s0 + u < nv ? __ldcg(ml + s0 + u) : make_float2(-INFINITY, 0.f);
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+                if (v[u].y > 0.f) mx = fmaxf(mx, v[u].x);
         }
         float num[E];
 #pragma unroll
         for (int e = 0; e < E; ++e) num[e] = 0.f;
         float den = 0.f;
-        for (int s = 0; s < nv; ++s) {
-            const float2 v = ml[s];
-            if (!(v.y > 0.f)) continue;
-            const float w = __expf(v.x - mx);
-            den = __fadd_rn(den, __fmul_rn(w, v.y));
-            const float *o = P.o_part + (((size_t)m * dm.Hq + h) * nsa + s) * DH;
+        for (int s0 = 0; s0 < nv; s0 += 4) {
+            float2 v[4];
+            float o[4][E];
 #pragma unroll
-            for (int e = 0; e < E; ++e) num[e] = __fadd_rn(num[e], __fmul_rn(w, o[lane + 32 * e]));
+            for (int u = 0; u < 4; ++u) {
+                const bool in = s0 + u < nv;
+                v[u] = in ? __ldcg(ml + s0 + u) : make_float2(-INFINITY, 0.f);
+#pragma unroll
+                for (int e = 0; e < E; ++e) o[u][e] = in ? __ldcg(ob + (size_t)(s0 + u) * DH + 32 * e) : 0.f;
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                if (!(v[u].y > 0.f)) continue;  // the row saw no key in this split
+                const float w = __expf(v[u].x - mx);
+                den = __fadd_rn(den, __fmul_rn(w, v[u].y));
+#pragma unroll
+                for (int e = 0; e < E; ++e) num[e] = __fadd_rn(num[e], __fmul_rn(w, o[u][e]));
+            }
         }
         bf16 *dst = P.attn + ((size_t)m * dm.Hq + h) * DH;
 #pragma unroll
@@ -698,11 +820,18 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
         // ---------------- compute group (warps 2-7)
         const int ct = tid - 64, cw = warp - 2;
         uint32_t li = 0;
+        unsigned long long *tr = P.trace ? P.trace + 4ull * P.cta_off[blockIdx.x] : nullptr;
         for (int i = 0; i < n_my; ++i) {
             const MKItem it = my[i];
+            if (tr && ct == 0) {
+                const unsigned long long now = globaltimer_ns();
+                if (i > 0) tr[4 * (i - 1) + 3] = now;
+                tr[4 * i] = now;
+            }
             if (ct == 0) s_flag = wait_deps(P, it) ? 1 : 0;
             bar_compute();
             if (!s_flag) break;
+            if (tr && ct == 0) tr[4 * i + 1] = tr[4 * i + 2] = globaltimer_ns();
             if (it.op == MK_EMBED) {
                 do_embed(P, it.a, cw, lane);
                 bar_compute();
@@ -715,9 +844,17 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 if (ct == 0) s_rms[0] = row_rms(P, m);
                 bar_compute();
                 const float rs = s_rms[0];
-                for (int f = ct; f < P.dm.H; f += CT)
-                    P.x_ro[(size_t)r * P.dm.H + f] =
-                        f2bf(__fmul_rn(bf2f(P.final_norm[f]), rbf(__fmul_rn(bf2f(P.h[(size_t)m * P.dm.H + f]), rs))));
+                for (int c8 = ct; c8 < P.dm.H / 8; c8 += CT) {
+                    const uint4 hv = __ldcg(reinterpret_cast<const uint4 *>(P.h + (size_t)m * P.dm.H) + c8);
+                    const uint4 gv = __ldg(reinterpret_cast<const uint4 *>(P.final_norm) + c8);
+                    const bf16 *he = reinterpret_cast<const bf16 *>(&hv);
+                    const bf16 *ge = reinterpret_cast<const bf16 *>(&gv);
+                    uint4 o;
+                    bf16 *oe = reinterpret_cast<bf16 *>(&o);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) oe[e] = f2bf(__fmul_rn(bf2f(ge[e]), rbf(__fmul_rn(bf2f(he[e]), rs))));
+                    reinterpret_cast<uint4 *>(P.x_ro + (size_t)r * P.dm.H)[c8] = o;
+                }
             } else if (it.op == MK_ATTN) {
                 const int bl = it.a, g = it.b, s = it.c;
                 const int b = P.pd.b0 + bl;
@@ -728,6 +865,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                         attn_split<64>(P, it.layer, bl, g, s, uni, ct, cw, lane);
                 }
                 bar_compute();
+                if (tr && ct == 0) tr[4 * i + 2] = globaltimer_ns();
                 int *c = ctr(P, it.layer, P.cl.att + bl * P.dm.Hkv + g);
                 if (ct == 0) {
                     __threadfence();
@@ -779,6 +917,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 }
                 ++li;
                 bar_compute();
+                if (tr && ct == 0) tr[4 * i + 2] = globaltimer_ns();
                 int *c = ctr(P, l, P.cl.lin[lin] + t);
                 if (ct == 0) {
                     __threadfence();
@@ -816,6 +955,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 }
             }
         }
+        if (tr && ct == 0 && n_my > 0) tr[4 * (n_my - 1) + 3] = globaltimer_ns();
     }
     tc_fence_before();
     __syncthreads();
@@ -905,7 +1045,7 @@ void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int
 
 size_t mk_union_bytes(int bn, int head_dim) {
     const size_t b = (size_t)ATOMS * bn * 128;
-    const size_t att = (size_t)ATT_SPLIT * (head_dim + 8) * 2 * 2;
+    const size_t att = (size_t)ATT_SPLIT * (head_dim + 8) * 2 * 2 + (ATT_SPLIT / PAGE) * sizeof(int);
     return std::max(b, att);
 }
 
@@ -956,6 +1096,7 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
     P.att_splits_alloc = L.att_splits_alloc;
     P.att_scale = (float)(1.0 / std::sqrt((double)L.dm.d));
     P.status = L.status;
+    P.trace = L.trace;
     P.abort = L.abort;
     P.bn = ((L.pd.M + 31) / 32) * 32;
     if (P.bn > MAX_ROWS || L.pd.M > MAX_ROWS) return cudaErrorInvalidValue;

@@ -91,6 +91,7 @@ struct pbd_ctx {
     float2 *ml_part;
     float *tile_max;
     int *tile_arg;
+    unsigned long long *trace;  // per-item timestamps of pbd_trace_pass
     int *ids, *draft_ids, *verify_ids, *first_id, *status, *cnt;  // cnt[0] = abort flag
     CounterLayout cl;
     Sched sched[N_PK];
@@ -162,7 +163,7 @@ bool valid_config(const pbd_config *cfg, std::string *why) {
         return bad("q/k/v widths must tile by 128 and the attention width by 256");
     if (k.intermediate % 256) return bad("intermediate must be a multiple of 256");
     if (k.vocab % 128) return bad("vocab must be a multiple of 128");
-    if (k.lora_rank < 1 || k.lora_rank > 32) return bad("lora_rank must be in [1, 32]");
+    if (k.lora_rank != 8 && k.lora_rank != 16) return bad("lora_rank must be 8 or 16");
     if (k.page_size != PAGE) return bad("page_size must be 16");
     if (k.block_D < 1 || k.block_D > 64) return bad("block_D must be in [1, 64]");
     if (k.max_batch < 1 || k.max_batch > 64) return bad("max_batch must be in [1, 64]");
@@ -277,6 +278,7 @@ size_t layout(pbd_ctx *c, void *base) {
     c->ml_part = (float2 *)bp.take(sizeof(float2) * (size_t)RA * Hq * c->n_splits);
     c->tile_max = (float *)bp.take(sizeof(float) * (size_t)(V / TILE_ROWS) * c->ro_alloc);
     c->tile_arg = (int *)bp.take(sizeof(int) * (size_t)(V / TILE_ROWS) * c->ro_alloc);
+    c->trace = (unsigned long long *)bp.take(sizeof(unsigned long long) * 4 * c->items_cap);
     return bp.off + ALIGN;
 }
 
@@ -967,6 +969,35 @@ pbd_status pbd_time_pass(pbd_ctx *c, int32_t kind, int32_t iters, double *h_ms_p
         CK(cudaMemcpy(Ls.data(), c->s.L, sizeof(int) * c->batch, cudaMemcpyDeviceToHost));
         *h_bytes_per_launch = pass_bytes(c, kind, Ls);
     }
+    return check_device(c);
+}
+
+pbd_status pbd_trace_pass(pbd_ctx *c, int32_t kind, int32_t *h_items, uint64_t *h_trace, int32_t cap, int32_t *h_n) {
+    if (!c || !h_items || !h_trace || !h_n) return fail(c, PBD_ERR_INVALID_ARG, "null argument");
+    if (kind < 0 || kind > 2) return fail(c, PBD_ERR_INVALID_ARG, "kind in [0,2]");
+    if (c->phase != PH_READY) return fail(c, PBD_ERR_STATE, "tracing needs a prefilled or committed state");
+    const PassDesc pd = block_pass(c, kind);
+    std::vector<MKItem> items;
+    std::vector<int> off;
+    mk_build_schedule(c->dm, pd, decode_splits(c), c->grid, &items, &off);
+    if ((int)items.size() > cap) return fail(c, PBD_ERR_CAPACITY, "%zu items exceed cap %d", items.size(), cap);
+    CK(launch_build_ids(pd, kind == PK_DRAFT ? 0 : (kind == PK_VERIFY ? 1 : 2), c->s.pending, c->draft_ids, c->D,
+                        c->ids, c->st));
+    CK(cudaMemsetAsync(c->trace, 0, sizeof(unsigned long long) * 4 * items.size(), c->st));
+    CK(cudaMemsetAsync(c->cnt, 0, sizeof(int) * (size_t)(c->cl.total + 1), c->st));
+    MKLaunch L = make_launch(c, pd, kind);
+    L.trace = c->trace;
+    CK(launch_pass_kernel(L, c->st));
+    CK(cudaMemcpyAsync(h_trace, c->trace, sizeof(unsigned long long) * 4 * items.size(), cudaMemcpyDeviceToHost,
+                       c->st));
+    CK(cudaStreamSynchronize(c->st));
+    for (size_t i = 0; i < items.size(); ++i) {
+        h_items[4 * i] = items[i].op | (items[i].lin << 8) | (items[i].layer << 16);
+        h_items[4 * i + 1] = items[i].a;
+        h_items[4 * i + 2] = items[i].b;
+        h_items[4 * i + 3] = items[i].c;
+    }
+    *h_n = (int32_t)items.size();
     return check_device(c);
 }
 

@@ -112,6 +112,7 @@ struct MKLaunch {
     float2 *ml_part;
     int att_splits_alloc;
     int *status, *abort;
+    unsigned long long *trace = nullptr;  // optional per-item timestamps
 };
 
 int mk_grid_size();

@@ -92,6 +92,8 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     L.pbd_version.restype = C.c_char_p
     L.pbd_bench_rounds.argtypes = [P, I32, I32, I32, P, P, P]
     L.pbd_time_pass.argtypes = [P, I32, I32, P, P]
+    L.pbd_trace_pass.argtypes = [P, I32, P, P, I32, P]
+    L.pbd_trace_pass.restype = C.c_int
     L.pbd_bench_rounds.restype = C.c_int
     L.pbd_time_pass.restype = C.c_int
     L.pbd_op_linear_workspace_bytes.restype = C.c_size_t
@@ -343,6 +345,15 @@ class Engine:
             fp = forced_n_seq.data_ptr()
         self._call(self.lib.pbd_bench_rounds, mode, warmup, steps, fp, ms.ctypes.data, launches.ctypes.data)
         return float(ms[0]), float(ms[1]), float(ms[2]), float(ms[3]), int(launches[0])
+
+    def pbd_trace_pass(self, kind: int, cap: int = 400000):
+        """(items [n, 4] int32 {op|lin<<8|layer<<16, a, b, c}, stamps [n, 4] uint64 ns) of one traced pass."""
+        items = np.zeros(cap * 4, np.int32)
+        tr = np.zeros(cap * 4, np.uint64)
+        n = np.zeros(1, np.int32)
+        self._call(self.lib.pbd_trace_pass, kind, items.ctypes.data, tr.ctypes.data, cap, n.ctypes.data)
+        k = int(n[0])
+        return items[: 4 * k].reshape(k, 4), tr[: 4 * k].reshape(k, 4)
 
     def pbd_time_pass(self, kind: int, iters: int):
         """(ms per launch, algorithmic bytes per launch) of the persistent pass kernel timed alone
