@@ -64,6 +64,7 @@ __device__ __forceinline__ int ld_relaxed(const int *p) {
 __device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
 struct MKParams {
+    CUtensorMap kmap, vmap;  // paged K / V cache as [rows of 128 dims] x d, box {64, 16}, 128-byte swizzle
     Dims dm;
     PassDesc pd;
     const MKItem *items;
@@ -454,15 +455,50 @@ __device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, i
     }
 }
 
-// ---- attention: one (sequence, KV head, 128-key split) on the compute group
+// ---- attention
 
-__device__ __forceinline__ uint32_t ldu32(const void *p) { return *reinterpret_cast<const uint32_t *>(p); }
+// Attention split staging layout in the union buffer: K then V, each DH/64 sub-tiles of
+// [128 keys x 128 bytes] in the 128-byte swizzle layout (16-byte chunk c of key n at
+// (c ^ (n & 7)) * 16), exactly as the tiled TMA writes them.
+constexpr int ATT_SUB_BYTES = ATT_SPLIT * 128;
 
+__device__ __forceinline__ uint32_t sw128(int row, int colb) {
+    return (uint32_t)(row * 128 + ((((colb >> 4) ^ (row & 7)) << 4) | (colb & 15)));
+}
+
+// TMA loads of the pages of one attention split (thread 0 of the compute group).
+// stage 0: pages entirely below the cached length L (written by earlier passes: prefetched
+// before the item's inputs are ready); stage 1: pages holding this pass's block rows.
+// Returns the bytes of the chosen pages; issues the copies only when `issue` is set.
+__device__ uint32_t attn_pages(const MKParams &P, int layer, int bl, int g, int s, int stage, uint8_t *smem,
+                               uint64_t *bar, bool issue) {
+    const int b = P.pd.b0 + bl;
+    const int L = P.L[b], T = L + P.pd.R, k0 = s * ATT_SPLIT;
+    const int subs = P.dm.d / 64;
+    uint32_t bytes = 0;
+    for (int p = 0; p < ATT_SPLIT / PAGE; ++p) {
+        const int kp0 = k0 + p * PAGE;
+        if (kp0 >= T || kp0 / PAGE >= P.kv.pages_per_seq) continue;
+        const bool cached = kp0 + PAGE <= L;
+        if (cached != (stage == 0)) continue;
+        bytes += (uint32_t)subs * 2u * PAGE * 128u;
+        if (!issue) continue;
+        const int phys = P.kv.page_table[b * P.kv.pages_per_seq + kp0 / PAGE];
+        const int row0 = ((layer * P.kv.n_pages + phys) * P.dm.Hkv + g) * PAGE;
+        for (int sub = 0; sub < subs; ++sub) {
+            tma_load_2d(smem + sub * ATT_SUB_BYTES + p * PAGE * 128, &P.kmap, sub * 64, row0, bar);
+            tma_load_2d(smem + (subs + sub) * ATT_SUB_BYTES + p * PAGE * 128, &P.vmap, sub * 64, row0, bar);
+        }
+    }
+    return bytes;
+}
+
+// One (sequence, KV head, 128-key split) on the compute group, after its K/V pages landed in
+// `smem` (stages 0 and 1 of attn_pages) and `bar` completed phase `parity`.
 template <int DH>
-__device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, int g, int s, uint8_t *smem, int ct, int cw,
-                           int lane) {
-    constexpr int KSTR = DH + 8, VSTR = DH + 8;
-    constexpr int NT = ATT_SPLIT / 8, KS = DH / 16, DT = DH / 8;
+__device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, int g, int s, uint8_t *smem,
+                                        uint64_t *bar, uint32_t parity, int ct, int cw, int lane) {
+    constexpr int NT = ATT_SPLIT / 8, KS = DH / 16, DT = DH / 8, SUBS = DH / 64;
     const Dims &dm = P.dm;
     const int b = P.pd.b0 + bl;
     const int L = P.L[b];
@@ -472,38 +508,19 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
     const int grp = dm.Hq / dm.Hkv;
     const int QV = R * grp;
     const int n_mt = (QV + 15) / 16;
-    bf16 *sK = reinterpret_cast<bf16 *>(smem);
-    __half *sV = reinterpret_cast<__half *>(smem + ATT_SPLIT * KSTR * 2);
-    int *s_page = reinterpret_cast<int *>(smem + ATT_SPLIT * KSTR * 2 + ATT_SPLIT * VSTR * 2);
-    const size_t layer_off = (size_t)layer * P.kv.n_pages * dm.Hkv * PAGE * DH;
-    const bf16 *kc = static_cast<const bf16 *>(P.kv.k), *vc = static_cast<const bf16 *>(P.kv.v);
-    // physical pages of the split (-1: beyond the keys of this pass or the reserved pages)
-    if (ct < ATT_SPLIT / PAGE) {
-        const int kp = k0 + ct * PAGE;
-        s_page[ct] = (kp < T && kp / PAGE < P.kv.pages_per_seq) ? P.kv.page_table[b * P.kv.pages_per_seq + kp / PAGE]
-                                                               : -1;
+    uint8_t *sK = smem, *sV = smem + SUBS * ATT_SUB_BYTES;
+    // pages without keys of this pass were not loaded: zero their V rows (p = 0 there, and
+    // 0 * stale bits could be NaN); their K rows are masked
+    for (int idx = ct; idx < (ATT_SPLIT / PAGE) * PAGE * SUBS * 8; idx += CT) {
+        const int chunk = idx % 8, row = (idx / 8) % ATT_SPLIT, sub = idx / (8 * ATT_SPLIT);
+        const int kp0 = k0 + (row / PAGE) * PAGE;
+        if (kp0 >= T || kp0 / PAGE >= P.kv.pages_per_seq)
+            *reinterpret_cast<uint4 *>(sV + sub * ATT_SUB_BYTES + row * 128 + chunk * 16) = make_uint4(0, 0, 0, 0);
     }
-    bar_compute();
-    // every 16-byte chunk of K and V in flight at once (async copies, zero fill past the last key)
-    for (int idx = ct; idx < ATT_SPLIT * (DH / 8); idx += CT) {
-        const int kk = idx / (DH / 8), c = idx % (DH / 8);
-        const int kp = k0 + kk, page = s_page[kk / PAGE];
-        const bool ok = page >= 0 && kp < T;
-        const size_t off = ok ? layer_off + (((size_t)page * dm.Hkv + g) * PAGE + (kp % PAGE)) * DH + (size_t)c * 8 : 0;
-        const uint32_t nbytes = ok ? 16u : 0u;
-        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(sK + kk * KSTR + c * 8)),
-                     "l"(kc + off), "r"(nbytes)
-                     : "memory");
-        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(sV + kk * VSTR + c * 8)),
-                     "l"(vc + off), "r"(nbytes)
-                     : "memory");
-    }
-    asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
-    bar_compute();
-    // V to fp16 in place (same size, same padded layout)
-    for (int idx = ct; idx < ATT_SPLIT * (DH / 8); idx += CT) {
-        const int kk = idx / (DH / 8), c = idx % (DH / 8);
-        uint4 *p4 = reinterpret_cast<uint4 *>(sV + kk * VSTR + c * 8);
+    const bool landed = mbar_wait_mk(bar, parity, P, DEV_TIMEOUT_LOAD);
+    // V to fp16 in place (each 16-byte chunk independently; the swizzle layout is unchanged)
+    for (int idx = ct; idx < SUBS * ATT_SUB_BYTES / 16; idx += CT) {
+        uint4 *p4 = reinterpret_cast<uint4 *>(sV + idx * 16);
         const uint4 v4 = *p4;
         const bf16 *ve = reinterpret_cast<const bf16 *>(&v4);
         uint4 h4;
@@ -513,6 +530,7 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
         *p4 = h4;
     }
     bar_compute();
+    if (!landed) return;
     const int gq = lane >> 2, tq = lane & 3;
     const bool blk = P.pd.mask_mode == MASK_BLOCK_DRAFT;
     for (int mt = cw; mt < n_mt; mt += CT / 32) {
@@ -526,18 +544,24 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
 #pragma unroll
         for (int ks = 0; ks < KS; ++ks) {
             const int c = ks * 16 + 2 * tq;
-            qa[ks][0] = val0 ? ldu32(q0 + c) : 0u;
-            qa[ks][1] = val1 ? ldu32(q1 + c) : 0u;
-            qa[ks][2] = val0 ? ldu32(q0 + c + 8) : 0u;
-            qa[ks][3] = val1 ? ldu32(q1 + c + 8) : 0u;
+            qa[ks][0] = val0 ? __ldcg(reinterpret_cast<const unsigned *>(q0 + c)) : 0u;
+            qa[ks][1] = val1 ? __ldcg(reinterpret_cast<const unsigned *>(q1 + c)) : 0u;
+            qa[ks][2] = val0 ? __ldcg(reinterpret_cast<const unsigned *>(q0 + c + 8)) : 0u;
+            qa[ks][3] = val1 ? __ldcg(reinterpret_cast<const unsigned *>(q1 + c + 8)) : 0u;
         }
         float sc[NT][4];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
             sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
-            const bf16 *krow = sK + (nt * 8 + gq) * KSTR + 2 * tq;
+            const int n = nt * 8 + gq;
 #pragma unroll
-            for (int ks = 0; ks < KS; ++ks) mma_m16n8k16_bf16(sc[nt], qa[ks], ldu32(krow + ks * 16), ldu32(krow + ks * 16 + 8));
+            for (int ks = 0; ks < KS; ++ks) {
+                const int e = ks * 16 + 2 * tq;
+                const uint8_t *kb = sK + (e >> 6) * ATT_SUB_BYTES;
+                const uint32_t b0 = *reinterpret_cast<const uint32_t *>(kb + sw128(n, (e & 63) * 2));
+                const uint32_t b1 = *reinterpret_cast<const uint32_t *>(kb + sw128(n, ((e + 8) & 63) * 2));
+                mma_m16n8k16_bf16(sc[nt], qa[ks], b0, b1);
+            }
         }
         const int qp0 = L + i0, qp1 = L + i1;
         const float scale = P.att_scale;
@@ -577,46 +601,50 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
         l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
         l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
         l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-        float oc[DT][4];
-#pragma unroll
-        for (int dt = 0; dt < DT; ++dt) oc[dt][0] = oc[dt][1] = oc[dt][2] = oc[dt][3] = 0.f;
+        // P as fp16 A fragments (k-step = 16 keys); the fp32 scores are dead from here on
+        uint32_t pa[ATT_SPLIT / 16][4];
 #pragma unroll
         for (int kstep = 0; kstep < ATT_SPLIT / 16; ++kstep) {
-            uint32_t pa[4];
-            pa[0] = pack_half2(sc[2 * kstep][0], sc[2 * kstep][1]);
-            pa[1] = pack_half2(sc[2 * kstep][2], sc[2 * kstep][3]);
-            pa[2] = pack_half2(sc[2 * kstep + 1][0], sc[2 * kstep + 1][1]);
-            pa[3] = pack_half2(sc[2 * kstep + 1][2], sc[2 * kstep + 1][3]);
-            const int vrow = kstep * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-#pragma unroll
-            for (int dt = 0; dt < DT; dt += 2) {
-                const int vcol = dt * 8 + (lane >> 4) * 8;
-                const uint32_t addr = smem_u32(sV + vrow * VSTR + vcol);
-                uint32_t r0, r1, r2, r3;
-                asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-                             : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-                             : "r"(addr));
-                mma_m16n8k16_f16(oc[dt], pa, r0, r1);
-                mma_m16n8k16_f16(oc[dt + 1], pa, r2, r3);
-            }
+            pa[kstep][0] = pack_half2(sc[2 * kstep][0], sc[2 * kstep][1]);
+            pa[kstep][1] = pack_half2(sc[2 * kstep][2], sc[2 * kstep][3]);
+            pa[kstep][2] = pack_half2(sc[2 * kstep + 1][0], sc[2 * kstep + 1][1]);
+            pa[kstep][3] = pack_half2(sc[2 * kstep + 1][2], sc[2 * kstep + 1][3]);
         }
         const int nsa = P.att_splits_alloc;
-        if (val0) {
-            const int m = bl * R + i0;
-            float *dst = P.o_part + (((size_t)m * dm.Hq + h0) * nsa + s) * DH;
+        float *dst0 = val0 ? P.o_part + (((size_t)(bl * R + i0) * dm.Hq + h0) * nsa + s) * DH : nullptr;
+        float *dst1 = val1 ? P.o_part + (((size_t)(bl * R + i1) * dm.Hq + h1) * nsa + s) * DH : nullptr;
+        // O = P V in halves of the head dimension (keeps the accumulators at 32 registers)
 #pragma unroll
-            for (int dt = 0; dt < DT; ++dt)
-                *reinterpret_cast<float2 *>(dst + dt * 8 + 2 * tq) = make_float2(oc[dt][0], oc[dt][1]);
-            if (tq == 0) P.ml_part[((size_t)m * dm.Hq + h0) * nsa + s] = make_float2(m0, l0);
-        }
-        if (val1) {
-            const int m = bl * R + i1;
-            float *dst = P.o_part + (((size_t)m * dm.Hq + h1) * nsa + s) * DH;
+        for (int half = 0; half < 2; ++half) {
+            float oc[DT / 2][4];
 #pragma unroll
-            for (int dt = 0; dt < DT; ++dt)
-                *reinterpret_cast<float2 *>(dst + dt * 8 + 2 * tq) = make_float2(oc[dt][2], oc[dt][3]);
-            if (tq == 0) P.ml_part[((size_t)m * dm.Hq + h1) * nsa + s] = make_float2(m1, l1);
+            for (int dt = 0; dt < DT / 2; ++dt) oc[dt][0] = oc[dt][1] = oc[dt][2] = oc[dt][3] = 0.f;
+#pragma unroll
+            for (int kstep = 0; kstep < ATT_SPLIT / 16; ++kstep) {
+                const int vrow = kstep * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+#pragma unroll
+                for (int dt = 0; dt < DT / 2; dt += 2) {
+                    const int vcol = (half * (DT / 2) + dt) * 8 + (lane >> 4) * 8;
+                    const uint32_t addr = smem_u32(sV + (vcol >> 6) * ATT_SUB_BYTES + sw128(vrow, (vcol & 63) * 2));
+                    uint32_t r0, r1, r2, r3;
+                    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                                 : "r"(addr));
+                    mma_m16n8k16_f16(oc[dt], pa[kstep], r0, r1);
+                    mma_m16n8k16_f16(oc[dt + 1], pa[kstep], r2, r3);
+                }
+            }
+#pragma unroll
+            for (int dt = 0; dt < DT / 2; ++dt) {
+                const int col = (half * (DT / 2) + dt) * 8 + 2 * tq;
+                if (val0) *reinterpret_cast<float2 *>(dst0 + col) = make_float2(oc[dt][0], oc[dt][1]);
+                if (val1) *reinterpret_cast<float2 *>(dst1 + col) = make_float2(oc[dt][2], oc[dt][3]);
+            }
         }
+        if (val0 && tq == 0)
+            P.ml_part[((size_t)(bl * R + i0) * dm.Hq + h0) * nsa + s] = make_float2(m0, l0);
+        if (val1 && tq == 0)
+            P.ml_part[((size_t)(bl * R + i1) * dm.Hq + h1) * nsa + s] = make_float2(m1, l1);
     }
 }
 
@@ -727,7 +755,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *ring = base;
     uint8_t *uni = base + P.ring_bytes;  // activation tile / attention staging
-    __shared__ __align__(8) uint64_t full[MAX_SLOT], empty[MAX_SLOT], b_full, acc_full;
+    __shared__ __align__(8) uint64_t full[MAX_SLOT], empty[MAX_SLOT], b_full, acc_full, att_bar;
     __shared__ uint32_t tmem_slot;
     // compute-group flags: each is written by thread 0 and read by all after a barrier, and is
     // not written again before every thread has passed at least one more barrier
@@ -745,6 +773,9 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
         }
         mbar_init(&b_full, 1);
         mbar_init(&acc_full, 1);
+        mbar_init(&att_bar, 1);
+        prefetch_tensormap(&P.kmap);
+        prefetch_tensormap(&P.vmap);
         fence_mbarrier_init();
     }
     if (warp == 0) tmem_alloc(&tmem_slot, P.tmem_cols);
@@ -819,7 +850,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
     } else {
         // ---------------- compute group (warps 2-7)
         const int ct = tid - 64, cw = warp - 2;
-        uint32_t li = 0;
+        uint32_t li = 0, ai = 0;
         unsigned long long *tr = P.trace ? P.trace + 4ull * P.cta_off[blockIdx.x] : nullptr;
         for (int i = 0; i < n_my; ++i) {
             const MKItem it = my[i];
@@ -828,6 +859,12 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 if (i > 0) tr[4 * (i - 1) + 3] = now;
                 tr[4 * i] = now;
             }
+            const bool att_active = it.op == MK_ATTN && it.c * ATT_SPLIT < P.L[P.pd.b0 + it.a] + P.pd.R;
+            if (att_active && ct == 0) {
+                // pages below the cached length do not depend on this pass: fetch them now
+                mbar_expect_tx(&att_bar, attn_pages(P, it.layer, it.a, it.b, it.c, 0, uni, &att_bar, false));
+                attn_pages(P, it.layer, it.a, it.b, it.c, 0, uni, &att_bar, true);
+            }
             if (ct == 0) s_flag = wait_deps(P, it) ? 1 : 0;
             bar_compute();
             if (!s_flag) break;
@@ -835,10 +872,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
             if (it.op == MK_EMBED) {
                 do_embed(P, it.a, cw, lane);
                 bar_compute();
-                if (ct == 0) {
-                    __threadfence();
-                    atomicAdd(P.cnt + P.cl.embed, 1);
-                }
+                if (ct == 0) red_release_add(P.cnt + P.cl.embed, 1);
             } else if (it.op == MK_FINAL) {
                 const int r = it.a, m = it.b;
                 if (ct == 0) s_rms[0] = row_rms(P, m);
@@ -857,22 +891,24 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 }
             } else if (it.op == MK_ATTN) {
                 const int bl = it.a, g = it.b, s = it.c;
-                const int b = P.pd.b0 + bl;
-                if (s * ATT_SPLIT < P.L[b] + P.pd.R) {
+                if (att_active) {
+                    if (ct == 0) {
+                        // the block's pages were written by this pass's q|k|v reducers (generic
+                        // stores, acquired above); order them before the TMA reads
+                        fence_proxy_async_global();
+                        mbar_arrive_expect_tx(&att_bar, attn_pages(P, it.layer, bl, g, s, 1, uni, &att_bar, false));
+                        attn_pages(P, it.layer, bl, g, s, 1, uni, &att_bar, true);
+                    }
                     if (P.dm.d == 128)
-                        attn_split<128>(P, it.layer, bl, g, s, uni, ct, cw, lane);
+                        attn_split<128>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane);
                     else
-                        attn_split<64>(P, it.layer, bl, g, s, uni, ct, cw, lane);
+                        attn_split<64>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane);
+                    ++ai;
                 }
                 bar_compute();
                 if (tr && ct == 0) tr[4 * i + 2] = globaltimer_ns();
                 int *c = ctr(P, it.layer, P.cl.att + bl * P.dm.Hkv + g);
-                if (ct == 0) {
-                    __threadfence();
-                    const int old = atomicAdd(c, 1);
-                    __threadfence();
-                    s_red = (old == P.nsplit[bl] - 1) ? 1 : 0;
-                }
+                if (ct == 0) s_red = (atom_acq_rel_add(c, 1) == P.nsplit[bl] - 1) ? 1 : 0;
                 bar_compute();
                 if (s_red) {
                     if (P.dm.d == 128)
@@ -880,10 +916,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                     else
                         attn_combine<64>(P, bl, g, cw, lane);
                     bar_compute();
-                    if (ct == 0) {
-                        __threadfence();
-                        atomicAdd(c, 1);
-                    }
+                    if (ct == 0) red_release_add(c, 1);
                 }
             } else {
                 // ---- linear slice item: stage activations, MMA (warp 1), epilogue, split reduction
@@ -919,12 +952,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 bar_compute();
                 if (tr && ct == 0) tr[4 * i + 2] = globaltimer_ns();
                 int *c = ctr(P, l, P.cl.lin[lin] + t);
-                if (ct == 0) {
-                    __threadfence();
-                    const int old = atomicAdd(c, 1);
-                    __threadfence();
-                    s_red = (old == P.ks[lin] - 1) ? 1 : 0;
-                }
+                if (ct == 0) s_red = (atom_acq_rel_add(c, 1) == P.ks[lin] - 1) ? 1 : 0;
                 bar_compute();
                 if (s_red) {
                     // this CTA finished the tile last: reduce the slices and finish the step
@@ -948,9 +976,8 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                         reduce_residual(P, lin, l, t, cw, lane);
                     bar_compute();
                     if (ct == 0) {
-                        __threadfence();
-                        atomicAdd(c, 1);
-                        if (!lt && (lin == 1 || lin == 3)) atomicAdd(ctr(P, l, lin == 1 ? P.cl.res_o : P.cl.res_dn), 1);
+                        red_release_add(c, 1);
+                        if (!lt && (lin == 1 || lin == 3)) red_release_add(ctr(P, l, lin == 1 ? P.cl.res_o : P.cl.res_dn), 1);
                     }
                 }
             }
@@ -1045,7 +1072,7 @@ void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int
 
 size_t mk_union_bytes(int bn, int head_dim) {
     const size_t b = (size_t)ATOMS * bn * 128;
-    const size_t att = (size_t)ATT_SPLIT * (head_dim + 8) * 2 * 2 + (ATT_SPLIT / PAGE) * sizeof(int);
+    const size_t att = (size_t)2 * (head_dim / 64) * ATT_SUB_BYTES;
     return std::max(b, att);
 }
 
@@ -1053,6 +1080,8 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
     cudaError_t e = device_limits();
     if (e != cudaSuccess) return e;
     MKParams P;
+    P.kmap = *L.kmap;
+    P.vmap = *L.vmap;
     P.dm = L.dm;
     P.pd = L.pd;
     P.items = L.items;

@@ -97,6 +97,7 @@ struct pbd_ctx {
     Sched sched[N_PK];
     SeqState s;
     CUtensorMap maps[N_BN];  // x_ro, per box height
+    CUtensorMap kmap, vmap;  // paged K and V caches
     // host state
     int batch = 0, max_new = 0;
     std::vector<int> prompt_lens;
@@ -286,6 +287,11 @@ pbd_status make_maps(pbd_ctx *c) {
     for (int i = 0; i < N_BN; ++i)
         if (!encode_bf16_map(&c->maps[i], c->x_ro, c->ro_alloc, c->cfg.hidden, BN_CHOICES[i]))
             return fail(c, PBD_ERR_CUDA, "tensor map encode failed (box rows %d)", BN_CHOICES[i]);
+    // K and V caches seen as rows of head_dim values: (layer, page, kv head, token) -> one row
+    const int kv_rows = c->cfg.n_layers * c->n_pages * c->cfg.n_kv_heads * PAGE;
+    if (!encode_bf16_map(&c->kmap, c->kv.k, kv_rows, c->cfg.head_dim, PAGE) ||
+        !encode_bf16_map(&c->vmap, c->kv.v, kv_rows, c->cfg.head_dim, PAGE))
+        return fail(c, PBD_ERR_CUDA, "KV tensor map encode failed");
     return PBD_OK;
 }
 
@@ -407,6 +413,8 @@ pbd_status upload_schedule(pbd_ctx *c, int kind, const PassDesc &pd, const std::
 MKLaunch make_launch(pbd_ctx *c, const PassDesc &pd, int kind) {
     MKLaunch L;
     const pbd_config &k = c->cfg;
+    L.kmap = &c->kmap;
+    L.vmap = &c->vmap;
     L.dm = c->dm;
     L.pd = pd;
     L.grid = c->grid;

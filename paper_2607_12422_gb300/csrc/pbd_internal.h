@@ -84,6 +84,7 @@ struct CounterLayout {
 };
 
 struct MKLaunch {
+    const CUtensorMap *kmap, *vmap;  // paged K / V cache, box {64 dims, 16 tokens}
     Dims dm;
     PassDesc pd;
     int grid;
