@@ -179,10 +179,12 @@ pbd_status pbd_time_pass(pbd_ctx *ctx, int32_t kind, int32_t iters, double *h_ms
 
 /* Timeline of one pass of the persistent kernel (a profiling aid; the paper's Appendix A.5 profiles
  * draft and verify forward latency).  On a prefilled context, runs one draft (kind 0), verify (1)
- * or plain-decoding (2) pass without advancing the state, recording for every work item four
- * %globaltimer stamps in ns: start, inputs complete, main work done, end.  h_items receives per
- * item {op | lin << 8 | layer << 16, a, b, c} (see the schedule description in the library),
- * h_trace the stamps, both in the schedule's order; at most `cap` items; *h_n the item count. */
+ * or plain-decoding (2) pass without advancing the state, recording for every work item eight
+ * %globaltimer stamps in ns: start, inputs complete, main work done, end, then per item kind
+ * (linear: operand staged, accumulator ready, completion counted, reduction done; attention:
+ * K/V landed, V converted, completion counted, merge done; 0 when not reached).  h_items
+ * receives per item {op | lin << 8 | layer << 16, a, b, c}, h_trace the stamps [n, 8], both in
+ * the schedule's order; at most `cap` items; *h_n the item count. */
 pbd_status pbd_trace_pass(pbd_ctx *ctx, int32_t kind, int32_t *h_items, uint64_t *h_trace, int32_t cap,
                           int32_t *h_n);
 

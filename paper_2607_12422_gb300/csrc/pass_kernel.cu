@@ -497,7 +497,8 @@ __device__ uint32_t attn_pages(const MKParams &P, int layer, int bl, int g, int 
 // `smem` (stages 0 and 1 of attn_pages) and `bar` completed phase `parity`.
 template <int DH>
 __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, int g, int s, uint8_t *smem,
-                                        uint64_t *bar, uint32_t parity, int ct, int cw, int lane) {
+                                        uint64_t *bar, uint32_t parity, int ct, int cw, int lane,
+                                        unsigned long long *stamp) {
     constexpr int NT = ATT_SPLIT / 8, KS = DH / 16, DT = DH / 8, SUBS = DH / 64;
     const Dims &dm = P.dm;
     const int b = P.pd.b0 + bl;
@@ -518,6 +519,7 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
             *reinterpret_cast<uint4 *>(sV + sub * ATT_SUB_BYTES + row * 128 + chunk * 16) = make_uint4(0, 0, 0, 0);
     }
     const bool landed = mbar_wait_mk(bar, parity, P, DEV_TIMEOUT_LOAD);
+    if (stamp && ct == 0) stamp[4] = globaltimer_ns();
     // V to fp16 in place (each 16-byte chunk independently; the swizzle layout is unchanged)
     for (int idx = ct; idx < SUBS * ATT_SUB_BYTES / 16; idx += CT) {
         uint4 *p4 = reinterpret_cast<uint4 *>(sV + idx * 16);
@@ -530,6 +532,7 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
         *p4 = h4;
     }
     bar_compute();
+    if (stamp && ct == 0) stamp[5] = globaltimer_ns();
     if (!landed) return;
     const int gq = lane >> 2, tq = lane & 3;
     const bool blk = P.pd.mask_mode == MASK_BLOCK_DRAFT;
@@ -851,13 +854,13 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
         // ---------------- compute group (warps 2-7)
         const int ct = tid - 64, cw = warp - 2;
         uint32_t li = 0, ai = 0;
-        unsigned long long *tr = P.trace ? P.trace + 4ull * P.cta_off[blockIdx.x] : nullptr;
+        unsigned long long *tr = P.trace ? P.trace + 8ull * P.cta_off[blockIdx.x] : nullptr;
         for (int i = 0; i < n_my; ++i) {
             const MKItem it = my[i];
             if (tr && ct == 0) {
                 const unsigned long long now = globaltimer_ns();
-                if (i > 0) tr[4 * (i - 1) + 3] = now;
-                tr[4 * i] = now;
+                if (i > 0) tr[8 * (i - 1) + 3] = now;
+                tr[8 * i] = now;
             }
             const bool att_active = it.op == MK_ATTN && it.c * ATT_SPLIT < P.L[P.pd.b0 + it.a] + P.pd.R;
             if (att_active && ct == 0) {
@@ -868,7 +871,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
             if (ct == 0) s_flag = wait_deps(P, it) ? 1 : 0;
             bar_compute();
             if (!s_flag) break;
-            if (tr && ct == 0) tr[4 * i + 1] = tr[4 * i + 2] = globaltimer_ns();
+            if (tr && ct == 0) tr[8 * i + 1] = tr[8 * i + 2] = globaltimer_ns();
             if (it.op == MK_EMBED) {
                 do_embed(P, it.a, cw, lane);
                 bar_compute();
@@ -900,15 +903,18 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                         attn_pages(P, it.layer, bl, g, s, 1, uni, &att_bar, true);
                     }
                     if (P.dm.d == 128)
-                        attn_split<128>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane);
+                        attn_split<128>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane,
+                                        tr ? tr + 8 * i : nullptr);
                     else
-                        attn_split<64>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane);
+                        attn_split<64>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane,
+                                       tr ? tr + 8 * i : nullptr);
                     ++ai;
                 }
                 bar_compute();
-                if (tr && ct == 0) tr[4 * i + 2] = globaltimer_ns();
+                if (tr && ct == 0) tr[8 * i + 2] = globaltimer_ns();
                 int *c = ctr(P, it.layer, P.cl.att + bl * P.dm.Hkv + g);
                 if (ct == 0) s_red = (atom_acq_rel_add(c, 1) == P.nsplit[bl] - 1) ? 1 : 0;
+                if (tr && ct == 0) tr[8 * i + 6] = tr[8 * i + 7] = globaltimer_ns();
                 bar_compute();
                 if (s_red) {
                     if (P.dm.d == 128)
@@ -917,6 +923,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                         attn_combine<64>(P, bl, g, cw, lane);
                     bar_compute();
                     if (ct == 0) red_release_add(c, 1);
+                    if (tr && ct == 0) tr[8 * i + 7] = globaltimer_ns();
                 }
             } else {
                 // ---- linear slice item: stage activations, MMA (warp 1), epilogue, split reduction
@@ -925,11 +932,13 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 fence_proxy_async();
                 bar_compute();
                 if (ct == 0) mbarrier_arrive_one(&b_full);
+                if (tr && ct == 0) tr[8 * i + 4] = globaltimer_ns();
                 const bool lt = t >= P.n_main[lin] / TILE_ROWS;
                 const int rows_valid = lt ? P.lora_rows[lin] : TILE_ROWS;
                 if (warp >= 4) {
                     const int quarter = warp - 4;
                     const bool have = mbar_wait_mk(&acc_full, li & 1, P, DEV_TIMEOUT_MMA);
+                    if (tr && warp == 4 && lane == 0) tr[8 * i + 5] = globaltimer_ns();
                     tc_fence_after();
                     if (have) {
                         const int row = quarter * 32 + lane;
@@ -950,9 +959,10 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 }
                 ++li;
                 bar_compute();
-                if (tr && ct == 0) tr[4 * i + 2] = globaltimer_ns();
+                if (tr && ct == 0) tr[8 * i + 2] = globaltimer_ns();
                 int *c = ctr(P, l, P.cl.lin[lin] + t);
                 if (ct == 0) s_red = (atom_acq_rel_add(c, 1) == P.ks[lin] - 1) ? 1 : 0;
+                if (tr && ct == 0) tr[8 * i + 6] = tr[8 * i + 7] = globaltimer_ns();
                 bar_compute();
                 if (s_red) {
                     // this CTA finished the tile last: reduce the slices and finish the step
@@ -979,10 +989,11 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                         red_release_add(c, 1);
                         if (!lt && (lin == 1 || lin == 3)) red_release_add(ctr(P, l, lin == 1 ? P.cl.res_o : P.cl.res_dn), 1);
                     }
+                    if (tr && ct == 0) tr[8 * i + 7] = globaltimer_ns();
                 }
             }
         }
-        if (tr && ct == 0 && n_my > 0) tr[4 * (n_my - 1) + 3] = globaltimer_ns();
+        if (tr && ct == 0 && n_my > 0) tr[8 * (n_my - 1) + 3] = globaltimer_ns();
     }
     tc_fence_before();
     __syncthreads();

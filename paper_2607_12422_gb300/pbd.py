@@ -347,13 +347,13 @@ class Engine:
         return float(ms[0]), float(ms[1]), float(ms[2]), float(ms[3]), int(launches[0])
 
     def pbd_trace_pass(self, kind: int, cap: int = 400000):
-        """(items [n, 4] int32 {op|lin<<8|layer<<16, a, b, c}, stamps [n, 4] uint64 ns) of one traced pass."""
+        """(items [n, 4] int32 {op|lin<<8|layer<<16, a, b, c}, stamps [n, 8] uint64 ns) of one traced pass."""
         items = np.zeros(cap * 4, np.int32)
-        tr = np.zeros(cap * 4, np.uint64)
+        tr = np.zeros(cap * 8, np.uint64)
         n = np.zeros(1, np.int32)
         self._call(self.lib.pbd_trace_pass, kind, items.ctypes.data, tr.ctypes.data, cap, n.ctypes.data)
         k = int(n[0])
-        return items[: 4 * k].reshape(k, 4), tr[: 4 * k].reshape(k, 4)
+        return items[: 4 * k].reshape(k, 4), tr[: 8 * k].reshape(k, 8)
 
     def pbd_time_pass(self, kind: int, iters: int):
         """(ms per launch, algorithmic bytes per launch) of the persistent pass kernel timed alone

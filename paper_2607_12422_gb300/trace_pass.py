@@ -38,6 +38,17 @@ def summarize(items, tr):
         out["phases"][name] = {"items": int(sel.sum()), "wait_us_med": float(np.median(wait)),
                                "work_us_med": float(np.median(work)), "post_us_med": float(np.median(post)),
                                "item_us_max": float((t[sel, 3] - t[sel, 0]).max())}
+        # sub-stamps 4..7 (0 = not reached): linear = operand staged, accumulator ready, counted,
+        # reduced; attention = K/V landed, V converted, counted, merged
+        sub = {}
+        labels = (("staged", "acc_ready", "counted", "reduced") if name not in ("attn",)
+                  else ("landed", "converted", "counted", "merged"))
+        for j, lab in enumerate(labels):
+            ok = sel & (tr[:, 4 + j] > 0)
+            if ok.any():
+                sub[lab + "_us_med"] = float(np.median(t[ok, 4 + j] - t[ok, 1]))
+        if sub:
+            out["phases"][name]["since_deps"] = sub
         ends[name] = {int(l): float(t[sel & (layer == l), 3].max()) for l in np.unique(layer[sel])}
     # per-layer span of each phase: end of this phase minus end of the previous phase in the layer
     prev = {"qkv": None, "attn": "qkv", "o": "attn", "gate_up": "o", "down": "gate_up"}
