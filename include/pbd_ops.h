@@ -29,6 +29,49 @@ size_t pbd_op_linear_workspace_bytes(int32_t M, int32_t K, int32_t N, int32_t r)
 pbd_status pbd_op_linear(int32_t M, int32_t K, int32_t N, int32_t r, float scale, const void *d_x, const void *d_w,
                          const void *d_a, const void *d_b, void *d_y, void *d_ws, size_t ws_bytes, void *d_stream);
 
+/* Bytes of the library's own device scratch behind pbd_op_linear_static, per device. */
+#define PBD_OP_LINEAR_STATIC_SCRATCH_BYTES (16u << 20)
+
+/* pbd_op_linear without a workspace.  This entry point has no counterpart in the paper: it is
+ * an integration aid.  It computes exactly what pbd_op_linear computes, with the same kernels
+ * and the same fixed-order sums, so for the same inputs the two give the same y.
+ *
+ * Who it is for: callers that cannot hand the library device memory.  For example a caller
+ * that sits behind an interface which passes only its input and output tensors, a process whose
+ * device memory is entirely owned by another allocator, or a loop that must not call cudaMalloc
+ * or cudaFree because those calls can synchronise the device.  Such a caller gets a call that
+ * never allocates or frees device memory (no cudaMalloc, cudaFree, stream-ordered or library
+ * allocation of any kind).
+ *
+ * Where the scratch lives: a fixed array of PBD_OP_LINEAR_STATIC_SCRATCH_BYTES (16 MiB) in the
+ * library's device code, one per device, created when the CUDA runtime loads that code on the
+ * device.  Its address is looked up the first time this function is called with a device current
+ * (also the time the kernels' attributes are set); make that first call on each device before
+ * any stream capture begins.
+ *
+ * Size limit: the call needs 2048 + (N/128 + (r > 0)) * (K/64) * 16384 + 4 * s * M * (N + r)
+ * bytes, s = K/256 when K is a multiple of 256 and 1 otherwise (the re-tiled weight, the
+ * adapter rows and the fp32 split-K partial sums).  Larger problems return PBD_ERR_CAPACITY
+ * before anything is launched, and the message gives both sizes; use pbd_op_linear for them.
+ * Within 16 MiB fit, for instance, an N = 6144, K = 1024 weight with r = 16 up to M = 39, and
+ * an N = 1024, K = 3072 weight with r = 16 up to M = 194.
+ *
+ * Zeroing: every call clears, on d_stream, the parts of the scratch that must start at zero
+ * (the kernel's status word and the adapter's row tile); everything else is overwritten before
+ * it is read, so a call never sees an earlier call's data.
+ *
+ * Concurrency: all calls on one device share the same scratch.  Two calls whose work can
+ * overlap in time on the device (different streams without an ordering between them, or
+ * several host threads with their own streams) race on it and can produce wrong results.
+ * Issue them on one stream, or order the streams.
+ *
+ * Arguments as pbd_op_linear, without d_ws and ws_bytes; the work runs on the current device
+ * and d_stream must belong to it.  Returns PBD_ERR_INVALID_ARG for unsupported sizes or null
+ * pointers, PBD_ERR_CAPACITY when the scratch is too small, PBD_ERR_CUDA when a runtime call
+ * fails (message from pbd_op_last_error()). */
+pbd_status pbd_op_linear_static(int32_t M, int32_t K, int32_t N, int32_t r, float scale, const void *d_x,
+                                const void *d_w, const void *d_a, const void *d_b, void *d_y, void *d_stream);
+
 /* Workspace bytes pbd_op_lm_head_argmax needs (0 if unsupported). */
 size_t pbd_op_lm_head_workspace_bytes(int32_t M, int32_t H, int32_t V);
 

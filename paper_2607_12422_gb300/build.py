@@ -17,7 +17,7 @@ BUILD_DIR = os.path.join(HERE, "_build")
 LIB_DIR = os.path.join(HERE, "lib")
 LIB = os.path.join(LIB_DIR, "libpbd.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["linear_tc.cu", "pass_kernel.cu", "ops.cu", "ops_api.cu", "pbd.cu"]
+SOURCES = ["linear_tc.cu", "pass_kernel.cu", "ops.cu", "ops_api.cu", "op_linear_static.cu", "pbd.cu"]
 HEADERS = ["common.cuh", "pbd_internal.h"]
 
 

@@ -176,3 +176,7 @@ pbd_status pbd_op_lm_head_argmax(int32_t M, int32_t H, int32_t V, const void *d_
 const char *pbd_op_last_error(void) { return g_op_err.c_str(); }
 
 }  // extern "C"
+
+namespace pbd {
+void op_record_error(const char *msg) { g_op_err = msg; }
+}  // namespace pbd

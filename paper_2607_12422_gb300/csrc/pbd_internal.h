@@ -187,4 +187,7 @@ bool encode_bf16_map(CUtensorMap *map, const void *base, int rows, int cols, int
 // Per-instantiation kernel attributes (dynamic shared memory), set once before any capture.
 cudaError_t configure_linear_kernels();
 
+// Records the message pbd_op_last_error() returns on this thread.
+void op_record_error(const char *msg);
+
 }  // namespace pbd

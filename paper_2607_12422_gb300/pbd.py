@@ -103,6 +103,8 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     L.pbd_op_lm_head_workspace_bytes.argtypes = [I32, I32, I32]
     L.pbd_op_lm_head_argmax.argtypes = [I32, I32, I32, P, P, P, P, P, C.c_size_t, P]
     L.pbd_op_last_error.restype = C.c_char_p
+    L.pbd_op_linear_static.argtypes = [I32, I32, I32, I32, C.c_float, P, P, P, P, P, P]
+    L.pbd_op_linear_static.restype = C.c_int
     for name in ("pbd_create", "pbd_destroy", "pbd_prefill", "pbd_draft_block", "pbd_verify_block",
                  "pbd_accept_commit", "pbd_decode_step", "pbd_generate", "pbd_get_state", "pbd_get_tokens",
                  "pbd_read_kv", "pbd_sync", "pbd_op_linear", "pbd_op_lm_head_argmax"):
@@ -137,6 +139,26 @@ def pbd_op_linear(x, W, A=None, B=None, scale: float = 2.0):
         raise PbdError(s, L.pbd_op_last_error().decode())
     torch.cuda.synchronize(x.device)
     del buf
+    return y
+
+
+def pbd_op_linear_static(x, W, A=None, B=None, scale: float = 2.0, y=None, sync: bool = True):
+    """pbd_op_linear through the entry point that takes no workspace (the library's own static
+    scratch); y [M, N] bf16 is the caller's output tensor (allocated here when not given)."""
+    import torch
+    L = load()
+    M, K = x.shape
+    N = W.shape[0]
+    r = A.shape[0] if (A is not None and B is not None) else 0
+    if y is None:
+        y = torch.empty(M, N, dtype=torch.bfloat16, device=x.device)
+    st = torch.cuda.current_stream(x.device).cuda_stream
+    s = L.pbd_op_linear_static(M, K, N, r, scale, x.data_ptr(), W.data_ptr(), _ptr(A) if r else None,
+                               _ptr(B) if r else None, y.data_ptr(), st)
+    if s != PBD_OK:
+        raise PbdError(s, L.pbd_op_last_error().decode())
+    if sync:
+        torch.cuda.synchronize(x.device)
     return y
 
 
