@@ -314,27 +314,29 @@ __device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int 
 }
 
 // reducer of the adapter tile: u = bf16(sum of slices), kept as fp32 values
-__device__ __noinline__ void reduce_lora(const MKParams &P, int lin, int ct) {
+__device__ __noinline__ void reduce_lora(const MKParams &P, int lin, int ct, int m0, int mstep) {
     const int M = P.pd.M, lr = P.lora_rows[lin], n0 = P.n_main[lin];
-    for (int q = ct; q < M * lr; q += CT) {
-        const int m = q / lr, j = q % lr;
+    const int nrow = m0 < M ? (M - m0 + mstep - 1) / mstep : 0;
+    for (int q = ct; q < nrow * lr; q += CT) {
+        const int m = m0 + (q / lr) * mstep, j = q % lr;
         const int f[1] = {n0 + j};
         float s[1];
-        sum_parts<1, 4>(P, lin, m, f, s);
-        P.red_lora[lin][q] = rbf(s[0]);
+        sum_parts<1, 8>(P, lin, m, f, s);
+        P.red_lora[lin][(size_t)m * lr + j] = rbf(s[0]);
     }
 }
 
 // q|k|v tile: adapter delta, bf16, per-head RMSNorm + RoPE for q and k, store q / paged K, V
 template <int DH>
-__device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, int cw, int lane) {
+__device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, int cw, int lane, int m0, int mstep) {
     constexpr int E = DH / 32;
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r;
     const int heads_per_tile = TILE_ROWS / DH;
     const bf16 *lb = P.lora_b[0] + (size_t)layer * P.lb_stride[0];
-    for (int it = cw; it < M * heads_per_tile; it += CT / 32) {
-        const int m = it / heads_per_tile, hh = it % heads_per_tile;
+    const int nrow = m0 < M ? (M - m0 + mstep - 1) / mstep : 0;
+    for (int it = cw; it < nrow * heads_per_tile; it += CT / 32) {
+        const int m = m0 + (it / heads_per_tile) * mstep, hh = it % heads_per_tile;
         const int fbase = tile * TILE_ROWS + hh * DH;
         const int qw = dm.Hq * DH, kvw = dm.Hkv * DH;
         const int kind = fbase < qw ? 0 : (fbase < qw + kvw ? 1 : 2);
@@ -347,7 +349,7 @@ __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, 
         float u[MAX_RANK];
         if (P.pd.adapter) load_u(P.red_lora[0] + (size_t)m * P.lora_rows[0] + kind * r, r, u);
         float y[E];
-        sum_parts<E, 4>(P, 0, m, f, y);
+        sum_parts<E, 8>(P, 0, m, f, y);
 #pragma unroll
         for (int j = 0; j < E; ++j) {
             if (P.pd.adapter) y[j] = __fadd_rn(y[j], __fmul_rn(dm.lora_scale, lora_dot_f(u, lb + (size_t)f[j] * r, r)));
@@ -397,11 +399,12 @@ __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, 
 }
 
 // o or down tile: adapter delta, residual add into h, per-tile sum of squares
-__device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int layer, int tile, int cw, int lane) {
+__device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int layer, int tile, int cw, int lane, int m0,
+                                             int mstep) {
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r, H = dm.H, nt = H / TILE_ROWS;
     const bf16 *lb = P.lora_b[lin] + (size_t)layer * P.lb_stride[lin];
-    for (int m = cw; m < M; m += CT / 32) {
+    for (int m = m0 + cw * mstep; m < M; m += (CT / 32) * mstep) {
         int f[4];
         float hv[4], acc[4];
 #pragma unroll
@@ -411,7 +414,7 @@ __device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int lay
         }
         float u[MAX_RANK];
         if (P.pd.adapter) load_u(P.red_lora[lin] + (size_t)m * P.lora_rows[lin], r, u);
-        sum_parts<4, 4>(P, lin, m, f, acc);
+        sum_parts<4, 8>(P, lin, m, f, acc);
         float v[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
@@ -425,11 +428,11 @@ __device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int lay
 }
 
 // gate|up tile (rows 0-63 gate features 64t.., rows 64-127 up features 64t..): SiLU(gate)*up
-__device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, int cw, int lane) {
+__device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, int cw, int lane, int m0, int mstep) {
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r, I = dm.I;
     const bf16 *lb = P.lora_b[2] + (size_t)layer * P.lb_stride[2];
-    for (int m = cw; m < M; m += CT / 32) {
+    for (int m = m0 + cw * mstep; m < M; m += (CT / 32) * mstep) {
         // partial rows: gate j = lane, lane+32 at tile rows j; up at tile rows 64 + j
         const int f[4] = {tile * TILE_ROWS + lane, tile * TILE_ROWS + lane + 32, tile * TILE_ROWS + 64 + lane,
                           tile * TILE_ROWS + 96 + lane};
@@ -438,7 +441,7 @@ __device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, i
             load_u(P.red_lora[2] + (size_t)m * P.lora_rows[2], r, ug);
             load_u(P.red_lora[2] + (size_t)m * P.lora_rows[2] + r, r, uu);
         }
-        sum_parts<4, 4>(P, 2, m, f, s);
+        sum_parts<4, 8>(P, 2, m, f, s);
 #pragma unroll
         for (int e = 0; e < 2; ++e) {
             const int a = tile * 64 + lane + 32 * e;  // act feature
@@ -499,7 +502,10 @@ template <int DH>
 __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, int g, int s, uint8_t *smem,
                                         uint64_t *bar, uint32_t parity, int ct, int cw, int lane,
                                         unsigned long long *stamp) {
-    constexpr int NT = ATT_SPLIT / 8, KS = DH / 16, DT = DH / 8, SUBS = DH / 64;
+    // each warp takes one 16-row query tile and one half of the split's keys; the halves are
+    // separate partial results (m, l, O) that the merge combines like splits
+    constexpr int NT = ATT_SPLIT / 8 / ATT_SUBS, KS = DH / 16, DT = DH / 8, SUBS = DH / 64;
+    constexpr int HALF = ATT_SPLIT / ATT_SUBS;
     const Dims &dm = P.dm;
     const int b = P.pd.b0 + bl;
     const int L = P.L[b];
@@ -536,7 +542,8 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
     if (!landed) return;
     const int gq = lane >> 2, tq = lane & 3;
     const bool blk = P.pd.mask_mode == MASK_BLOCK_DRAFT;
-    for (int mt = cw; mt < n_mt; mt += CT / 32) {
+    for (int unit = cw; unit < n_mt * ATT_SUBS; unit += CT / 32) {
+        const int mt = unit / ATT_SUBS, half = unit % ATT_SUBS, kb = half * HALF;
         const int qv0 = mt * 16 + gq, qv1 = qv0 + 8;
         const bool val0 = qv0 < QV, val1 = qv1 < QV;
         const int i0 = val0 ? qv0 / grp : 0, i1 = val1 ? qv1 / grp : 0;
@@ -556,7 +563,7 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
             sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
-            const int n = nt * 8 + gq;
+            const int n = kb + nt * 8 + gq;
 #pragma unroll
             for (int ks = 0; ks < KS; ++ks) {
                 const int e = ks * 16 + 2 * tq;
@@ -573,7 +580,7 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
         for (int nt = 0; nt < NT; ++nt) {
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
-                const int kp = k0 + nt * 8 + 2 * tq + e;
+                const int kp = k0 + kb + nt * 8 + 2 * tq + e;
                 const bool vis0 = val0 && kp < T && (kp <= qp0 || (blk && i0 >= 1 && kp > L));
                 const bool vis1 = val1 && kp < T && (kp <= qp1 || (blk && i1 >= 1 && kp > L));
                 sc[nt][e] = vis0 ? __fmul_rn(sc[nt][e], scale) : -INFINITY;
@@ -605,17 +612,18 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
         l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
         l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
         // P as fp16 A fragments (k-step = 16 keys); the fp32 scores are dead from here on
-        uint32_t pa[ATT_SPLIT / 16][4];
+        uint32_t pa[HALF / 16][4];
 #pragma unroll
-        for (int kstep = 0; kstep < ATT_SPLIT / 16; ++kstep) {
+        for (int kstep = 0; kstep < HALF / 16; ++kstep) {
             pa[kstep][0] = pack_half2(sc[2 * kstep][0], sc[2 * kstep][1]);
             pa[kstep][1] = pack_half2(sc[2 * kstep][2], sc[2 * kstep][3]);
             pa[kstep][2] = pack_half2(sc[2 * kstep + 1][0], sc[2 * kstep + 1][1]);
             pa[kstep][3] = pack_half2(sc[2 * kstep + 1][2], sc[2 * kstep + 1][3]);
         }
         const int nsa = P.att_splits_alloc;
-        float *dst0 = val0 ? P.o_part + (((size_t)(bl * R + i0) * dm.Hq + h0) * nsa + s) * DH : nullptr;
-        float *dst1 = val1 ? P.o_part + (((size_t)(bl * R + i1) * dm.Hq + h1) * nsa + s) * DH : nullptr;
+        const int sub = s * ATT_SUBS + half;  // index of this partial result
+        float *dst0 = val0 ? P.o_part + (((size_t)(bl * R + i0) * dm.Hq + h0) * nsa + sub) * DH : nullptr;
+        float *dst1 = val1 ? P.o_part + (((size_t)(bl * R + i1) * dm.Hq + h1) * nsa + sub) * DH : nullptr;
         // O = P V in halves of the head dimension (keeps the accumulators at 32 registers)
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
@@ -623,8 +631,8 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
 #pragma unroll
             for (int dt = 0; dt < DT / 2; ++dt) oc[dt][0] = oc[dt][1] = oc[dt][2] = oc[dt][3] = 0.f;
 #pragma unroll
-            for (int kstep = 0; kstep < ATT_SPLIT / 16; ++kstep) {
-                const int vrow = kstep * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+            for (int kstep = 0; kstep < HALF / 16; ++kstep) {
+                const int vrow = kb + kstep * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
 #pragma unroll
                 for (int dt = 0; dt < DT / 2; dt += 2) {
                     const int vcol = (half * (DT / 2) + dt) * 8 + (lane >> 4) * 8;
@@ -645,23 +653,24 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
             }
         }
         if (val0 && tq == 0)
-            P.ml_part[((size_t)(bl * R + i0) * dm.Hq + h0) * nsa + s] = make_float2(m0, l0);
+            P.ml_part[((size_t)(bl * R + i0) * dm.Hq + h0) * nsa + sub] = make_float2(m0, l0);
         if (val1 && tq == 0)
-            P.ml_part[((size_t)(bl * R + i1) * dm.Hq + h1) * nsa + s] = make_float2(m1, l1);
+            P.ml_part[((size_t)(bl * R + i1) * dm.Hq + h1) * nsa + sub] = make_float2(m1, l1);
     }
 }
 
 // merge the splits of (row, head) in split order; splits where the row saw no key are skipped
 template <int DH>
-__device__ __noinline__ void attn_combine(const MKParams &P, int bl, int g, int cw, int lane) {
+__device__ __noinline__ void attn_combine(const MKParams &P, int bl, int g, int cw, int lane, int p0, int pstep) {
     const Dims &dm = P.dm;
     const int R = P.pd.R, grp = dm.Hq / dm.Hkv;
     const int b = P.pd.b0 + bl;
     const int T = P.L[b] + R;
     const int nsa = P.att_splits_alloc;
-    const int nv = min(P.nsplit[bl], (T + ATT_SPLIT - 1) / ATT_SPLIT);  // splits computed in this pass
+    // partial results computed in this pass: ATT_SUBS per split that holds a key
+    const int nv = min(P.nsplit[bl], (T + ATT_SPLIT - 1) / ATT_SPLIT) * ATT_SUBS;
     constexpr int E = DH / 32;
-    for (int it = cw; it < R * grp; it += CT / 32) {
+    for (int it = p0 + cw * pstep; it < R * grp; it += (CT / 32) * pstep) {
         const int i = it / grp, h = g * grp + it % grp;
         const int m = bl * R + i;
         const float2 *ml = P.ml_part + ((size_t)m * dm.Hq + h) * nsa;
@@ -704,11 +713,17 @@ __device__ __noinline__ void attn_combine(const MKParams &P, int bl, int g, int 
     }
 }
 
-// wait for every tile of linear `lin` that holds output features [f0, f1)
+// Attention merge mode of a (sequence, head) with nsp splits: shared by all splits when they sit
+// on distinct CTAs (nsp <= grid), else done by the last split; and the count that marks it done.
+__device__ __forceinline__ bool att_shared_merge(int nsp) { return nsp <= (int)gridDim.x; }
+__device__ __forceinline__ int att_done(int nsp) { return att_shared_merge(nsp) ? 2 * nsp : nsp + 1; }
+
+// wait for every tile of linear `lin` that holds output features [f0, f1): each of its ks
+// slices counts once when stored and once when its rows are reduced
 __device__ bool wait_tiles(const MKParams &P, int layer, int lin, int f0, int f1) {
     const int off = P.cl.lin[lin];
     for (int t = f0 / TILE_ROWS; t <= (f1 - 1) / TILE_ROWS; ++t)
-        if (!spin_until(ctr(P, layer, off + t), P.ks[lin] + 1, P)) return false;
+        if (!spin_until(ctr(P, layer, off + t), 2 * P.ks[lin], P)) return false;
     return true;
 }
 
@@ -721,21 +736,22 @@ __device__ bool wait_deps(const MKParams &P, const MKItem &it) {
         switch (it.lin) {
             case 0:
                 if (l == 0) return spin_until(P.cnt + P.cl.embed, P.pd.M, P);
-                return spin_until(ctr(P, l - 1, P.cl.res_dn), dm.H / TILE_ROWS, P);
+                return spin_until(ctr(P, l - 1, P.cl.res_dn), dm.H / TILE_ROWS * P.ks[3], P);
             case 1: {
                 const int h0 = (s * KSLICE) / dm.d, h1 = (s * KSLICE + KSLICE - 1) / dm.d;
                 const int grp = dm.Hq / dm.Hkv;
                 for (int bl = 0; bl < P.pd.nb; ++bl)
                     for (int g = h0 / grp; g <= h1 / grp; ++g)
-                        if (!spin_until(ctr(P, l, P.cl.att + bl * dm.Hkv + g), P.nsplit[bl] + 1, P)) return false;
+                        if (!spin_until(ctr(P, l, P.cl.att + bl * dm.Hkv + g), att_done(P.nsplit[bl]), P))
+                            return false;
                 return true;
             }
-            case 2: return spin_until(ctr(P, l, P.cl.res_o), dm.H / TILE_ROWS, P);
+            case 2: return spin_until(ctr(P, l, P.cl.res_o), dm.H / TILE_ROWS * P.ks[1], P);
             default: {
                 // act features [256 s, 256 s + 256) live in gate|up tiles 4s..4s+3
                 const int t0 = (s * KSLICE) / 64, t1 = (s * KSLICE + KSLICE - 1) / 64;
                 for (int t = t0; t <= t1; ++t)
-                    if (!spin_until(ctr(P, l, P.cl.lin[2] + t), P.ks[2] + 1, P)) return false;
+                    if (!spin_until(ctr(P, l, P.cl.lin[2] + t), 2 * P.ks[2], P)) return false;
                 return true;
             }
         }
@@ -747,7 +763,7 @@ __device__ bool wait_deps(const MKParams &P, const MKItem &it) {
                wait_tiles(P, l, 0, qw + g * d, qw + (g + 1) * d) &&
                wait_tiles(P, l, 0, qw + kvw + g * d, qw + kvw + (g + 1) * d);
     }
-    if (it.op == MK_FINAL) return spin_until(ctr(P, dm.nl - 1, P.cl.res_dn), dm.H / TILE_ROWS, P);
+    if (it.op == MK_FINAL) return spin_until(ctr(P, dm.nl - 1, P.cl.res_dn), dm.H / TILE_ROWS * P.ks[3], P);
     return true;
 }
 
@@ -912,15 +928,30 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 }
                 bar_compute();
                 if (tr && ct == 0) tr[8 * i + 2] = globaltimer_ns();
+                // merge: when the (sequence, head)'s splits fit on distinct CTAs, every split waits for
+                // the others and merges pairs s, s + nsplit, ...; otherwise the last one merges all
                 int *c = ctr(P, it.layer, P.cl.att + bl * P.dm.Hkv + g);
-                if (ct == 0) s_red = (atom_acq_rel_add(c, 1) == P.nsplit[bl] - 1) ? 1 : 0;
+                const int nsp = P.nsplit[bl];
+                const bool shared_merge = att_shared_merge(nsp);
+                if (ct == 0) {
+                    if (shared_merge) {
+                        red_release_add(c, 1);
+                        s_ok = spin_until(c, nsp, P) ? 1 : 0;
+                        s_red = 1;
+                    } else {
+                        s_red = (atom_acq_rel_add(c, 1) == nsp - 1) ? 1 : 0;
+                        s_ok = 1;
+                    }
+                }
                 if (tr && ct == 0) tr[8 * i + 6] = tr[8 * i + 7] = globaltimer_ns();
                 bar_compute();
+                if (!s_ok) break;
                 if (s_red) {
+                    const int p0 = shared_merge ? s : 0, pstep = shared_merge ? nsp : 1;
                     if (P.dm.d == 128)
-                        attn_combine<128>(P, bl, g, cw, lane);
+                        attn_combine<128>(P, bl, g, cw, lane, p0, pstep);
                     else
-                        attn_combine<64>(P, bl, g, cw, lane);
+                        attn_combine<64>(P, bl, g, cw, lane, p0, pstep);
                     bar_compute();
                     if (ct == 0) red_release_add(c, 1);
                     if (tr && ct == 0) tr[8 * i + 7] = globaltimer_ns();
@@ -960,37 +991,39 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 ++li;
                 bar_compute();
                 if (tr && ct == 0) tr[8 * i + 2] = globaltimer_ns();
+                // The tile's slices are consecutive items of the round-robin schedule, so they sit on
+                // distinct CTAs that all reach them: each CTA announces its stored slice, waits for the
+                // others, then reduces rows s, s + ks, ... of the tile (s = its slice).
                 int *c = ctr(P, l, P.cl.lin[lin] + t);
-                if (ct == 0) s_red = (atom_acq_rel_add(c, 1) == P.ks[lin] - 1) ? 1 : 0;
-                if (tr && ct == 0) tr[8 * i + 6] = tr[8 * i + 7] = globaltimer_ns();
-                bar_compute();
-                if (s_red) {
-                    // this CTA finished the tile last: reduce the slices and finish the step
-                    if (!lt && P.pd.adapter && P.lora_rows[lin] > 0) {
-                        if (ct == 0)
-                            s_ok = spin_until(ctr(P, l, P.cl.lin[lin] + P.n_main[lin] / TILE_ROWS), P.ks[lin] + 1, P)
-                                       ? 1 : 0;
-                        bar_compute();
-                        if (!s_ok) break;
-                    }
-                    if (lt)
-                        reduce_lora(P, lin, ct);
-                    else if (lin == 0) {
-                        if (P.dm.d == 128)
-                            reduce_qkv<128>(P, l, t, cw, lane);
-                        else
-                            reduce_qkv<64>(P, l, t, cw, lane);
-                    } else if (lin == 2)
-                        reduce_gu(P, l, t, cw, lane);
-                    else
-                        reduce_residual(P, lin, l, t, cw, lane);
-                    bar_compute();
-                    if (ct == 0) {
-                        red_release_add(c, 1);
-                        if (!lt && (lin == 1 || lin == 3)) red_release_add(ctr(P, l, lin == 1 ? P.cl.res_o : P.cl.res_dn), 1);
-                    }
-                    if (tr && ct == 0) tr[8 * i + 7] = globaltimer_ns();
+                const int ks = P.ks[lin];
+                if (ct == 0) {
+                    red_release_add(c, 1);
+                    if (tr) tr[8 * i + 6] = globaltimer_ns();
+                    bool ok = spin_until(c, ks, P);
+                    // the adapter rows' u must be final before a main tile adds the delta
+                    if (ok && !lt && P.pd.adapter && P.lora_rows[lin] > 0)
+                        ok = spin_until(ctr(P, l, P.cl.lin[lin] + P.n_main[lin] / TILE_ROWS), 2 * ks, P);
+                    s_ok = ok ? 1 : 0;
                 }
+                bar_compute();
+                if (!s_ok) break;
+                if (lt)
+                    reduce_lora(P, lin, ct, s, ks);
+                else if (lin == 0) {
+                    if (P.dm.d == 128)
+                        reduce_qkv<128>(P, l, t, cw, lane, s, ks);
+                    else
+                        reduce_qkv<64>(P, l, t, cw, lane, s, ks);
+                } else if (lin == 2)
+                    reduce_gu(P, l, t, cw, lane, s, ks);
+                else
+                    reduce_residual(P, lin, l, t, cw, lane, s, ks);
+                bar_compute();
+                if (ct == 0) {
+                    red_release_add(c, 1);
+                    if (!lt && (lin == 1 || lin == 3)) red_release_add(ctr(P, l, lin == 1 ? P.cl.res_o : P.cl.res_dn), 1);
+                }
+                if (tr && ct == 0) tr[8 * i + 7] = globaltimer_ns();
             }
         }
         if (tr && ct == 0 && n_my > 0) tr[8 * (n_my - 1) + 3] = globaltimer_ns();
@@ -1107,6 +1140,8 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
         P.lora_rows[i] = L.lora_rows[i];
         P.K[i] = L.K[i];
         P.ks[i] = L.K[i] / KSLICE;
+        // a tile's K slices wait for one another, so each must sit on its own CTA
+        if (P.ks[i] > L.grid) return cudaErrorInvalidConfiguration;
         P.lora_b[i] = static_cast<const bf16 *>(L.lora_b[i]);
         P.lb_stride[i] = L.lb_stride[i];
         P.part[i] = L.part[i];

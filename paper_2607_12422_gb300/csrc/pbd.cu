@@ -162,7 +162,9 @@ bool valid_config(const pbd_config *cfg, std::string *why) {
     if (k.hidden % 256 || k.hidden > 4096) return bad("hidden must be a multiple of 256, at most 4096");
     if ((k.n_q_heads * k.head_dim) % 256 || ((k.n_q_heads + 2 * k.n_kv_heads) * k.head_dim) % 128)
         return bad("q/k/v widths must tile by 128 and the attention width by 256");
-    if (k.intermediate % 256) return bad("intermediate must be a multiple of 256");
+    if (k.intermediate % 256 || k.intermediate > 16384)
+        return bad("intermediate must be a multiple of 256, at most 16384");
+    if (k.n_q_heads * k.head_dim > 16384) return bad("n_q_heads * head_dim must be at most 16384");
     if (k.vocab % 128) return bad("vocab must be a multiple of 128");
     if (k.lora_rank != 8 && k.lora_rank != 16) return bad("lora_rank must be 8 or 16");
     if (k.page_size != PAGE) return bad("page_size must be 16");
@@ -275,8 +277,8 @@ size_t layout(pbd_ctx *c, void *base) {
                                         (lin_main(k, lin) + lin_lora(k, lin)));
         c->red_lora[lin] = (float *)bp.take(sizeof(float) * (size_t)RA * lin_lora(k, lin));
     }
-    c->o_part = (float *)bp.take(sizeof(float) * (size_t)RA * Hq * c->n_splits * d);
-    c->ml_part = (float2 *)bp.take(sizeof(float2) * (size_t)RA * Hq * c->n_splits);
+    c->o_part = (float *)bp.take(sizeof(float) * (size_t)RA * Hq * c->n_splits * ATT_SUBS * d);
+    c->ml_part = (float2 *)bp.take(sizeof(float2) * (size_t)RA * Hq * c->n_splits * ATT_SUBS);
     c->tile_max = (float *)bp.take(sizeof(float) * (size_t)(V / TILE_ROWS) * c->ro_alloc);
     c->tile_arg = (int *)bp.take(sizeof(int) * (size_t)(V / TILE_ROWS) * c->ro_alloc);
     c->trace = (unsigned long long *)bp.take(sizeof(unsigned long long) * 8 * c->items_cap);
@@ -458,7 +460,7 @@ MKLaunch make_launch(pbd_ctx *c, const PassDesc &pd, int kind) {
     L.ss = c->ss;
     L.o_part = c->o_part;
     L.ml_part = c->ml_part;
-    L.att_splits_alloc = c->n_splits;
+    L.att_splits_alloc = c->n_splits * ATT_SUBS;  // partial results per (row, head)
     L.status = c->status;
     L.abort = c->cnt;
     return L;

@@ -12,6 +12,7 @@ namespace pbd {
 
 constexpr int PAGE = 16;           // KV page length in tokens
 constexpr int ATT_SPLIT = 128;     // key positions per attention split (position-aligned)
+constexpr int ATT_SUBS = 2;        // partial results per split (its two 64-key halves)
 constexpr int PREFILL_ROWS = 64;   // rows per prefill chunk
 constexpr int KT = 64;             // K elements per 128-byte swizzle atom row (bf16)
 constexpr int TILE_ROWS = 128;     // output features per tensor-core tile

@@ -75,6 +75,7 @@ def main():
     ap.add_argument("--workload", default="qwen3-0.6b-b1-d16-p512-g256")
     ap.add_argument("--kind", default="verify", choices=["draft", "verify", "decode"])
     ap.add_argument("--repeat", type=int, default=3)
+    ap.add_argument("--dump", default="", help="also save the raw items and stamps to this .npz file")
     a = ap.parse_args()
     from paper_2607_12422_gb300 import pbd, synth
     W = synth.WORKLOADS[a.workload]
@@ -89,6 +90,8 @@ def main():
         items, tr = eng.pbd_trace_pass(kind)
         res = summarize(items, tr)
     res["workload"], res["kind"] = a.workload, a.kind
+    if a.dump:
+        np.savez(a.dump, items=items, stamps=tr)
     print(json.dumps(res, indent=1))
 
 
