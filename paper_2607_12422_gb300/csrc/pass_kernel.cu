@@ -40,8 +40,8 @@ namespace pbd {
 
 constexpr int MK_THREADS = 256;
 constexpr int CT = 192;            // compute-group threads (warps 2-7)
-constexpr int KSLICE = 256;        // K elements per linear item
-constexpr int ATOMS = KSLICE / KT; // 64-wide swizzle atoms per item
+constexpr int HALF_ATOMS = 4;      // 64-wide swizzle atoms of one operand staging round (K 256)
+constexpr int MAX_ATOMS = 8;       // atoms per linear item at most (K slice 512)
 constexpr int MAX_SLOT = 12;
 constexpr int MAX_ROWS = 256;
 
@@ -76,6 +76,8 @@ struct MKParams {
     const uint8_t *wt[4];      // tiled weights of layer 0; layer stride wt_stride[lin] bytes
     size_t wt_stride[4];
     int n_main[4], lora_rows[4], K[4], ks[4];
+    int katoms[4];             // 64-wide K atoms per item (the K slice is 64 * katoms wide)
+    int b_dbl;                 // the operand area holds a whole MAX_ATOMS item at once
     const bf16 *lora_b[4];     // fused adapter B of layer 0, [n_out][r]
     size_t lb_stride[4];       // elements per layer
     const bf16 *attn_norm, *mlp_norm, *q_norm, *k_norm, *final_norm, *mask_embed, *embed_tiled;
@@ -168,15 +170,20 @@ __device__ __forceinline__ float ldcg_bf(const bf16 *p) {
 
 // 1/sqrt(mean(h^2) + eps) of row m from its per-tile sums (tiles added in order)
 __device__ __forceinline__ float row_rms(const MKParams &P, int m) {
-    const int nt = P.dm.H / TILE_ROWS;
-    const float *s = P.ss + (size_t)m * nt;
-    float v[MAX_HT];
+    const int nt = P.dm.H / TILE_ROWS;  // even (H is a multiple of 256)
+    const float2 *s = reinterpret_cast<const float2 *>(P.ss + (size_t)m * nt);
+    float a = 0.f;
+    for (int t0 = 0; t0 < nt; t0 += 8) {
+        float2 v[4];
 #pragma unroll
-    for (int t = 0; t < MAX_HT; ++t) v[t] = t < nt ? __ldcg(s + t) : 0.f;
-    float a = v[0];
+        for (int u = 0; u < 4; ++u) v[u] = t0 + 2 * u < nt ? __ldcg(s + t0 / 2 + u) : make_float2(0.f, 0.f);
 #pragma unroll
-    for (int t = 1; t < MAX_HT; ++t)
-        if (t < nt) a = __fadd_rn(a, v[t]);
+        for (int u = 0; u < 4; ++u) {
+            if (t0 + 2 * u >= nt) break;
+            a = (t0 + u == 0) ? v[u].x : __fadd_rn(a, v[u].x);
+            a = __fadd_rn(a, v[u].y);
+        }
+    }
     return __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(__fdiv_rn(a, (float)P.dm.H), P.dm.eps)));
 }
 
@@ -269,35 +276,42 @@ __device__ __noinline__ void do_embed(const MKParams &P, int m, int cw, int lane
 // Activation tile of one linear item in the 128-byte swizzle layout: atom j (K columns
 // 64j..64j+63 of the slice) holds row m at m*128 bytes, 16-byte chunk c at (c ^ (m & 7)) * 16.
 // Row m of the q|k|v and gate|up inputs is RMSNorm(h_m) * gain, computed here on the fly.
-__device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int slice, uint8_t *sb, float *s_rms, int ct) {
+__device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int slice, uint8_t *sb, float *s_rms, int ct,
+                                     int a0, int na, bool need_rms) {
     constexpr int U = 4;  // chunks in flight per thread
     const int M = P.pd.M;
-    const int k0 = slice * KSLICE;
+    const int k0 = (slice * P.katoms[lin] + a0) * KT;
+    const int cpr = na * (KT / 8);  // 16-byte chunks per row
     const bool norm = (lin == 0 || lin == 2);
-    if (norm) {
-        for (int m = ct; m < M; m += CT) s_rms[m] = row_rms(P, m);
-        bar_compute();
-    }
     const bf16 *gain = lin == 0 ? P.attn_norm + (size_t)layer * P.dm.H : P.mlp_norm + (size_t)layer * P.dm.H;
     const bf16 *src = norm ? P.h : (lin == 1 ? P.attn : P.act);
     const int ld = norm ? P.dm.H : (lin == 1 ? P.dm.Hq * P.dm.d : P.dm.I);
-    const int chunks = M * (KSLICE / 8);
-    for (int q0 = ct; q0 < chunks; q0 += U * CT) {
-        uint4 xv[U], gv[U];
+    const int chunks = M * cpr;
+    uint4 xv[U], gv[U];
+    auto issue = [&](int q0) {
 #pragma unroll
         for (int u = 0; u < U; ++u) {
             const int q = q0 + u * CT;
             if (q < chunks) {
-                const int m = q / (KSLICE / 8), c = q % (KSLICE / 8);
+                const int m = q / cpr, c = q % cpr;
                 xv[u] = __ldcg(reinterpret_cast<const uint4 *>(src + (size_t)m * ld + k0 + c * 8));
                 if (norm) gv[u] = __ldg(reinterpret_cast<const uint4 *>(gain + k0 + c * 8));
             }
         }
+    };
+    // the first chunks are in flight while the rows' norm scales are computed
+    issue(ct);
+    if (norm && need_rms) {
+        for (int m = ct; m < M; m += CT) s_rms[m] = row_rms(P, m);
+        bar_compute();
+    }
+    for (int q0 = ct; q0 < chunks; q0 += U * CT) {
+        if (q0 != ct) issue(q0);
 #pragma unroll
         for (int u = 0; u < U; ++u) {
             const int q = q0 + u * CT;
             if (q >= chunks) break;
-            const int m = q / (KSLICE / 8), c = q % (KSLICE / 8);
+            const int m = q / cpr, c = q % cpr;
             const int atom = c >> 3, cc = c & 7;
             uint4 val = xv[u];
             if (norm) {
@@ -738,7 +752,8 @@ __device__ bool wait_deps(const MKParams &P, const MKItem &it) {
                 if (l == 0) return spin_until(P.cnt + P.cl.embed, P.pd.M, P);
                 return spin_until(ctr(P, l - 1, P.cl.res_dn), dm.H / TILE_ROWS * P.ks[3], P);
             case 1: {
-                const int h0 = (s * KSLICE) / dm.d, h1 = (s * KSLICE + KSLICE - 1) / dm.d;
+                const int w = P.katoms[1] * KT;
+                const int h0 = (s * w) / dm.d, h1 = (s * w + w - 1) / dm.d;
                 const int grp = dm.Hq / dm.Hkv;
                 for (int bl = 0; bl < P.pd.nb; ++bl)
                     for (int g = h0 / grp; g <= h1 / grp; ++g)
@@ -749,7 +764,8 @@ __device__ bool wait_deps(const MKParams &P, const MKItem &it) {
             case 2: return spin_until(ctr(P, l, P.cl.res_o), dm.H / TILE_ROWS * P.ks[1], P);
             default: {
                 // act features [256 s, 256 s + 256) live in gate|up tiles 4s..4s+3
-                const int t0 = (s * KSLICE) / 64, t1 = (s * KSLICE + KSLICE - 1) / 64;
+                const int w = P.katoms[3] * KT;
+                const int t0 = (s * w) / 64, t1 = (s * w + w - 1) / 64;
                 for (int t = t0; t <= t1; ++t)
                     if (!spin_until(ctr(P, l, P.cl.lin[2] + t), 2 * P.ks[2], P)) return false;
                 return true;
@@ -774,7 +790,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *ring = base;
     uint8_t *uni = base + P.ring_bytes;  // activation tile / attention staging
-    __shared__ __align__(8) uint64_t full[MAX_SLOT], empty[MAX_SLOT], b_full, acc_full, att_bar;
+    __shared__ __align__(8) uint64_t full[MAX_SLOT], empty[MAX_SLOT], b_full[2], b_empty, acc_full, att_bar;
     __shared__ uint32_t tmem_slot;
     // compute-group flags: each is written by thread 0 and read by all after a barrier, and is
     // not written again before every thread has passed at least one more barrier
@@ -790,7 +806,9 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
             mbar_init(&full[i], 1);
             mbar_init(&empty[i], 1);
         }
-        mbar_init(&b_full, 1);
+        mbar_init(&b_full[0], 1);
+        mbar_init(&b_full[1], 1);
+        mbar_init(&b_empty, 1);
         mbar_init(&acc_full, 1);
         mbar_init(&att_bar, 1);
         prefetch_tensormap(&P.kmap);
@@ -799,7 +817,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
     }
     if (warp == 0) tmem_alloc(&tmem_slot, P.tmem_cols);
     // zero the padding rows of the activation tile once (rows >= M are never written)
-    for (int q = tid; q < ATOMS * P.bn * 8; q += MK_THREADS) {
+    for (int q = tid; q < (P.b_dbl ? MAX_ATOMS : HALF_ATOMS) * P.bn * 8; q += MK_THREADS) {
         const int atom = q / (P.bn * 8), rem = q % (P.bn * 8), m = rem / 8;
         if (m >= P.pd.M) *reinterpret_cast<uint4 *>(uni + (size_t)atom * P.bn * 128 + rem * 16) = make_uint4(0, 0, 0, 0);
     }
@@ -821,9 +839,9 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 const uint32_t bytes = lt ? (uint32_t)P.lora_rows[lin] * 128u : (uint32_t)TILE_BYTES;
                 const int kts = P.K[lin] / KT;
                 const uint8_t *src = P.wt[lin] + P.wt_stride[lin] * it.layer +
-                                     ((size_t)it.a * kts + (size_t)it.b * ATOMS) * TILE_BYTES;
+                                     ((size_t)it.a * kts + (size_t)it.b * P.katoms[lin]) * TILE_BYTES;
                 bool ok = true;
-                for (int j = 0; j < ATOMS; ++j, ++kt) {
+                for (int j = 0; j < P.katoms[lin]; ++j, ++kt) {
                     const int slot = kt % P.nslot;
                     if (kt >= (uint32_t)P.nslot &&
                         !mbar_wait_mk(&empty[slot], ((kt / P.nslot) - 1) & 1, P, DEV_TIMEOUT_SLOT)) {
@@ -840,14 +858,25 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
         // ---------------- MMA issuer
         if (lane == 0) {
             const uint32_t idesc = idesc_bf16_f32(128, P.bn);
-            uint32_t kt = 0, li = 0;
+            uint32_t kt = 0, li = 0, l8 = 0;
             for (int i = 0; i < n_my; ++i) {
                 const MKItem it = my[i];
                 if (it.op != MK_LINEAR) continue;
-                if (!mbar_wait_mk(&b_full, li & 1, P, DEV_TIMEOUT_LOAD)) break;
+                const int na = P.katoms[it.lin];
+                if (!mbar_wait_mk(&b_full[0], li & 1, P, DEV_TIMEOUT_LOAD)) break;
                 tc_fence_after();
                 bool ok = true;
-                for (int j = 0; j < ATOMS; ++j, ++kt) {
+                for (int j = 0; j < na; ++j, ++kt) {
+                    if (j == HALF_ATOMS) {
+                        // second half of a wide slice: its operand is staged after the first
+                        // half's reads completed (same area) or was staged with it
+                        mma_commit(&b_empty);
+                        if (!mbar_wait_mk(&b_full[1], l8 & 1, P, DEV_TIMEOUT_LOAD)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                    }
                     const int slot = kt % P.nslot;
                     if (!mbar_wait_mk(&full[slot], (kt / P.nslot) & 1, P, DEV_TIMEOUT_LOAD)) {
                         ok = false;
@@ -855,7 +884,8 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                     }
                     tc_fence_after();
                     const uint64_t ad = sw128_kmajor_desc(ring + (size_t)slot * TILE_BYTES);
-                    const uint64_t bd = sw128_kmajor_desc(uni + (size_t)j * P.bn * 128);
+                    const int bj = (P.b_dbl || j < HALF_ATOMS) ? j : j - HALF_ATOMS;
+                    const uint64_t bd = sw128_kmajor_desc(uni + (size_t)bj * P.bn * 128);
 #pragma unroll
                     for (int kk = 0; kk < KT / 16; ++kk)
                         mma_bf16_ss(tmem, ad + 2ull * kk, bd + 2ull * kk, idesc, (j | kk) != 0 ? 1u : 0u);
@@ -864,12 +894,13 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 if (!ok) break;
                 mma_commit(&acc_full);
                 ++li;
+                if (na > HALF_ATOMS) ++l8;
             }
         }
     } else {
         // ---------------- compute group (warps 2-7)
         const int ct = tid - 64, cw = warp - 2;
-        uint32_t li = 0, ai = 0;
+        uint32_t li = 0, ai = 0, l8 = 0;
         unsigned long long *tr = P.trace ? P.trace + 8ull * P.cta_off[blockIdx.x] : nullptr;
         for (int i = 0; i < n_my; ++i) {
             const MKItem it = my[i];
@@ -959,10 +990,32 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
             } else {
                 // ---- linear slice item: stage activations, MMA (warp 1), epilogue, split reduction
                 const int lin = it.lin, l = it.layer, t = it.a, s = it.b;
-                build_b(P, lin, l, s, uni, s_rms, ct);
-                fence_proxy_async();
-                bar_compute();
-                if (ct == 0) mbarrier_arrive_one(&b_full);
+                const int na = P.katoms[lin];
+                if (na <= HALF_ATOMS || P.b_dbl) {
+                    build_b(P, lin, l, s, uni, s_rms, ct, 0, na, true);
+                    fence_proxy_async();
+                    bar_compute();
+                    if (ct == 0) {
+                        mbarrier_arrive_one(&b_full[0]);
+                        if (na > HALF_ATOMS) mbarrier_arrive_one(&b_full[1]);
+                    }
+                } else {
+                    // operand in two rounds through the same area
+                    build_b(P, lin, l, s, uni, s_rms, ct, 0, HALF_ATOMS, true);
+                    fence_proxy_async();
+                    bar_compute();
+                    if (ct == 0) {
+                        mbarrier_arrive_one(&b_full[0]);
+                        s_ok = mbar_wait_mk(&b_empty, l8 & 1, P, DEV_TIMEOUT_MMA) ? 1 : 0;
+                    }
+                    bar_compute();
+                    if (!s_ok) break;
+                    build_b(P, lin, l, s, uni, s_rms, ct, HALF_ATOMS, na - HALF_ATOMS, false);
+                    fence_proxy_async();
+                    bar_compute();
+                    if (ct == 0) mbarrier_arrive_one(&b_full[1]);
+                }
+                if (na > HALF_ATOMS) ++l8;
                 if (tr && ct == 0) tr[8 * i + 4] = globaltimer_ns();
                 const bool lt = t >= P.n_main[lin] / TILE_ROWS;
                 const int rows_valid = lt ? P.lora_rows[lin] : TILE_ROWS;
@@ -1088,7 +1141,7 @@ void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int
     const int n_main[4] = {nq, dm.H / TILE_ROWS, 2 * dm.I / TILE_ROWS, dm.H / TILE_ROWS};
     const int K[4] = {dm.H, dm.Hq * dm.d, dm.H, dm.I};
     auto linear = [&](int lin, int l) {
-        const int ks = K[lin] / KSLICE;
+        const int ks = K[lin] / (mk_slice_atoms(lin, K[lin]) * KT);
         if (pd.adapter)
             for (int s = 0; s < ks; ++s) push(MK_LINEAR, lin, l, n_main[lin], s, 0);
         for (int t = 0; t < n_main[lin]; ++t)
@@ -1114,8 +1167,12 @@ void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int
     for (size_t i = 0; i < all.size(); ++i) (*out)[fill[i % grid]++] = all[i];
 }
 
+// 64-wide K atoms per item of linear `lin`: gate|up takes 512-wide slices (half as many items,
+// so that one pass's gate|up items fit one per CTA), the others 256-wide
+int mk_slice_atoms(int lin, int K) { return (lin == 2 && K % (MAX_ATOMS * KT) == 0) ? MAX_ATOMS : HALF_ATOMS; }
+
 size_t mk_union_bytes(int bn, int head_dim) {
-    const size_t b = (size_t)ATOMS * bn * 128;
+    const size_t b = (size_t)HALF_ATOMS * bn * 128;
     const size_t att = (size_t)2 * (head_dim / 64) * ATT_SUB_BYTES;
     return std::max(b, att);
 }
@@ -1139,7 +1196,8 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
         P.n_main[i] = L.n_main[i];
         P.lora_rows[i] = L.lora_rows[i];
         P.K[i] = L.K[i];
-        P.ks[i] = L.K[i] / KSLICE;
+        P.katoms[i] = mk_slice_atoms(i, L.K[i]);
+        P.ks[i] = L.K[i] / (P.katoms[i] * KT);
         // a tile's K slices wait for one another, so each must sit on its own CTA
         if (P.ks[i] > L.grid) return cudaErrorInvalidConfiguration;
         P.lora_b[i] = static_cast<const bf16 *>(L.lora_b[i]);
@@ -1184,6 +1242,7 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
     if (P.nslot < 2) return cudaErrorInvalidValue;
     P.ring_bytes = P.nslot * TILE_BYTES;
     P.union_bytes = (int)uni;
+    P.b_dbl = (size_t)MAX_ATOMS * P.bn * 128 <= uni ? 1 : 0;
     const size_t dyn = (size_t)P.ring_bytes + uni + 1024;
     static size_t configured = 0;
     if (dyn > configured) {

@@ -122,6 +122,7 @@ void mk_counter_layout(const Dims &dm, int max_nb, CounterLayout *cl);
 void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int> &nsplit, int grid,
                        std::vector<MKItem> *out, std::vector<int> *off);
 size_t mk_union_bytes(int bn, int head_dim);
+int mk_slice_atoms(int lin, int K);  // 64-wide K atoms per work item of linear `lin`
 cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st);
 
 // ---- launchers (each returns cudaGetLastError()) ----
