@@ -43,6 +43,7 @@ constexpr int CT = 192;            // compute-group threads (warps 2-7)
 constexpr int HALF_ATOMS = 4;      // 64-wide swizzle atoms of one operand staging round (K 256)
 constexpr int MAX_ATOMS = 8;       // atoms per linear item at most (K slice 512)
 constexpr int MAX_SLOT = 12;
+constexpr int RING_SLOTS = 6;      // weight tiles in the ring (96 KiB)
 constexpr int MAX_ROWS = 256;
 
 // ------------------------------------------------------------------ device helpers
@@ -1238,7 +1239,9 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
     const size_t uni = mk_union_bytes(P.bn, L.dm.d);
     const size_t static_smem = 4096;
     const long avail = (long)g_smem_optin - (long)uni - 1024 - (long)static_smem;
-    P.nslot = (int)std::min<long>(MAX_SLOT, avail / TILE_BYTES);
+    // a shallow ring: what shared memory does not take stays L1 cache, which the compute warps
+    // stack frames, spills and read-only loads need more than the weight stream needs depth
+    P.nslot = (int)std::min<long>(RING_SLOTS, avail / TILE_BYTES);
     if (P.nslot < 2) return cudaErrorInvalidValue;
     P.ring_bytes = P.nslot * TILE_BYTES;
     P.union_bytes = (int)uni;
