@@ -43,7 +43,7 @@ constexpr int CT = 192;            // compute-group threads (warps 2-7)
 constexpr int HALF_ATOMS = 4;      // 64-wide swizzle atoms of one operand staging round (K 256)
 constexpr int MAX_ATOMS = 8;       // atoms per linear item at most (K slice 512)
 constexpr int MAX_SLOT = 12;
-constexpr int RING_SLOTS = 6;      // weight tiles in the ring (96 KiB)
+constexpr int RING_SLOTS = 4;      // weight tiles in the ring (64 KiB)
 constexpr int MAX_ROWS = 256;
 
 // ------------------------------------------------------------------ device helpers
