@@ -871,7 +871,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                     if (j == HALF_ATOMS) {
                         // second half of a wide slice: its operand is staged after the first
                         // half's reads completed (same area) or was staged with it
-                        mma_commit(&b_empty);
+                        if (!P.b_dbl) mma_commit(&b_empty);
                         if (!mbar_wait_mk(&b_full[1], l8 & 1, P, DEV_TIMEOUT_LOAD)) {
                             ok = false;
                             break;
@@ -992,14 +992,22 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 // ---- linear slice item: stage activations, MMA (warp 1), epilogue, split reduction
                 const int lin = it.lin, l = it.layer, t = it.a, s = it.b;
                 const int na = P.katoms[lin];
-                if (na <= HALF_ATOMS || P.b_dbl) {
+                if (na <= HALF_ATOMS) {
                     build_b(P, lin, l, s, uni, s_rms, ct, 0, na, true);
                     fence_proxy_async();
                     bar_compute();
-                    if (ct == 0) {
-                        mbarrier_arrive_one(&b_full[0]);
-                        if (na > HALF_ATOMS) mbarrier_arrive_one(&b_full[1]);
-                    }
+                    if (ct == 0) mbarrier_arrive_one(&b_full[0]);
+                } else if (P.b_dbl) {
+                    // wide slice, both halves fit: the first half's MMAs run while the second is staged
+                    build_b(P, lin, l, s, uni, s_rms, ct, 0, HALF_ATOMS, true);
+                    fence_proxy_async();
+                    bar_compute();
+                    if (ct == 0) mbarrier_arrive_one(&b_full[0]);
+                    build_b(P, lin, l, s, uni + (size_t)HALF_ATOMS * P.bn * 128, s_rms, ct, HALF_ATOMS,
+                            na - HALF_ATOMS, false);
+                    fence_proxy_async();
+                    bar_compute();
+                    if (ct == 0) mbarrier_arrive_one(&b_full[1]);
                 } else {
                     // operand in two rounds through the same area
                     build_b(P, lin, l, s, uni, s_rms, ct, 0, HALF_ATOMS, true);
