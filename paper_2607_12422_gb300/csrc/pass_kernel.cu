@@ -90,7 +90,6 @@ struct MKParams {
     // scratch
     float *part[4];
     int part_rows;
-    float *red_lora[4];
     bf16 *h, *q, *attn, *act, *x_ro;
     float *ss;                 // [rows][H/128]
     float *o_part;
@@ -162,7 +161,6 @@ __device__ __forceinline__ float tile_sumsq(const float (&v)[4]) {
 // With one CTA per SM only six compute warps hide memory latency, so every helper below issues
 // all of its independent loads before it consumes any; sums still run in one fixed order.
 // Data written by other CTAs during the pass is read with L2-only loads (never a stale L1 line).
-constexpr int MAX_HT = 32;     // 128-feature tiles of the hidden size (H <= 4096)
 constexpr int MAX_RANK = 16;   // adapter rank (8 or 16)
 
 __device__ __forceinline__ float ldcg_bf(const bf16 *p) {
@@ -188,17 +186,32 @@ __device__ __forceinline__ float row_rms(const MKParams &P, int m) {
     return __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(__fdiv_rn(a, (float)P.dm.H), P.dm.eps)));
 }
 
-// u[0..r) of row m: the bf16-rounded adapter intermediates x A^T (kept as fp32), r % 4 == 0
-__device__ __forceinline__ void load_u(const float *src, int r, float (&u)[MAX_RANK]) {
+// u[0..r) of row m for one adapter of linear `lin` (its rows c0 .. c0 + r - 1 in the adapter
+// tile): the bf16-rounded adapter intermediates x A^T, kept as fp32.  Summed here from the
+// adapter tile's K-slice partials (slices in order), so a main tile's reducer does not wait for
+// a separate reduction of the adapter tile.  Lane j < r sums u_j; the warp shares the vector.
+// Every lane of the warp calls it.
+__device__ __forceinline__ void lora_u(const MKParams &P, int lin, int m, int c0, int lane, float (&u)[MAX_RANK]) {
+    const int r = P.dm.r, ks = P.ks[lin];
+    const int nt = P.n_main[lin] + P.lora_rows[lin];
+    const float *p = P.part[lin] + (size_t)m * nt + P.n_main[lin] + c0 + lane;
+    const size_t stride = (size_t)P.part_rows * nt;
+    float a = 0.f;
+    if (lane < r) {
+        for (int s0 = 0; s0 < ks; s0 += 8) {
+            float v[8];
 #pragma unroll
-    for (int q = 0; q < MAX_RANK / 4; ++q) {
-        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (q * 4 < r) v = __ldcg(reinterpret_cast<const float4 *>(src) + q);
-        u[4 * q] = v.x;
-        u[4 * q + 1] = v.y;
-        u[4 * q + 2] = v.z;
-        u[4 * q + 3] = v.w;
+            for (int s = 0; s < 8; ++s) v[s] = s0 + s < ks ? __ldcg(p + (size_t)(s0 + s) * stride) : 0.f;
+#pragma unroll
+            for (int s = 0; s < 8; ++s) {
+                if (s0 + s >= ks) break;
+                a = (s0 + s == 0) ? v[s] : __fadd_rn(a, v[s]);
+            }
+        }
+        a = rbf(a);
     }
+#pragma unroll
+    for (int j = 0; j < MAX_RANK; ++j) u[j] = __shfl_sync(0xffffffffu, a, j);
 }
 
 // sum_j u_j * B[f, j] over j = 0..r-1 in order (B row: r bf16 values, r % 8 == 0)
@@ -328,19 +341,6 @@ __device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int 
     }
 }
 
-// reducer of the adapter tile: u = bf16(sum of slices), kept as fp32 values
-__device__ __noinline__ void reduce_lora(const MKParams &P, int lin, int ct, int m0, int mstep) {
-    const int M = P.pd.M, lr = P.lora_rows[lin], n0 = P.n_main[lin];
-    const int nrow = m0 < M ? (M - m0 + mstep - 1) / mstep : 0;
-    for (int q = ct; q < nrow * lr; q += CT) {
-        const int m = m0 + (q / lr) * mstep, j = q % lr;
-        const int f[1] = {n0 + j};
-        float s[1];
-        sum_parts<1, 8>(P, lin, m, f, s);
-        P.red_lora[lin][(size_t)m * lr + j] = rbf(s[0]);
-    }
-}
-
 // q|k|v tile: adapter delta, bf16, per-head RMSNorm + RoPE for q and k, store q / paged K, V
 template <int DH>
 __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, int cw, int lane, int m0, int mstep) {
@@ -362,7 +362,7 @@ __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, 
 #pragma unroll
         for (int j = 0; j < E; ++j) f[j] = fbase + lane + 32 * j;
         float u[MAX_RANK];
-        if (P.pd.adapter) load_u(P.red_lora[0] + (size_t)m * P.lora_rows[0] + kind * r, r, u);
+        if (P.pd.adapter) lora_u(P, 0, m, kind * r, lane, u);
         float y[E];
         sum_parts<E, 8>(P, 0, m, f, y);
 #pragma unroll
@@ -428,7 +428,7 @@ __device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int lay
             hv[e] = bf2f(ldcg_bf(P.h + (size_t)m * H + f[e]));
         }
         float u[MAX_RANK];
-        if (P.pd.adapter) load_u(P.red_lora[lin] + (size_t)m * P.lora_rows[lin], r, u);
+        if (P.pd.adapter) lora_u(P, lin, m, 0, lane, u);
         sum_parts<4, 8>(P, lin, m, f, acc);
         float v[4];
 #pragma unroll
@@ -453,8 +453,8 @@ __device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, i
                           tile * TILE_ROWS + 96 + lane};
         float ug[MAX_RANK], uu[MAX_RANK], s[4];
         if (P.pd.adapter) {
-            load_u(P.red_lora[2] + (size_t)m * P.lora_rows[2], r, ug);
-            load_u(P.red_lora[2] + (size_t)m * P.lora_rows[2] + r, r, uu);
+            lora_u(P, 2, m, 0, lane, ug);
+            lora_u(P, 2, m, r, lane, uu);
         }
         sum_parts<4, 8>(P, 2, m, f, s);
 #pragma unroll
@@ -1058,20 +1058,24 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 // others, then reduces rows s, s + ks, ... of the tile (s = its slice).
                 int *c = ctr(P, l, P.cl.lin[lin] + t);
                 const int ks = P.ks[lin];
+                if (lt) {
+                    // the adapter tile's partials are summed by the main tiles' reducers themselves
+                    if (ct == 0) red_release_add(c, 1);
+                    if (tr && ct == 0) tr[8 * i + 6] = tr[8 * i + 7] = globaltimer_ns();
+                    continue;
+                }
                 if (ct == 0) {
                     red_release_add(c, 1);
                     if (tr) tr[8 * i + 6] = globaltimer_ns();
                     bool ok = spin_until(c, ks, P);
-                    // the adapter rows' u must be final before a main tile adds the delta
-                    if (ok && !lt && P.pd.adapter && P.lora_rows[lin] > 0)
-                        ok = spin_until(ctr(P, l, P.cl.lin[lin] + P.n_main[lin] / TILE_ROWS), 2 * ks, P);
+                    // every slice of the adapter tile must be stored before a main tile adds the delta
+                    if (ok && P.pd.adapter && P.lora_rows[lin] > 0)
+                        ok = spin_until(ctr(P, l, P.cl.lin[lin] + P.n_main[lin] / TILE_ROWS), ks, P);
                     s_ok = ok ? 1 : 0;
                 }
                 bar_compute();
                 if (!s_ok) break;
-                if (lt)
-                    reduce_lora(P, lin, ct, s, ks);
-                else if (lin == 0) {
+                if (lin == 0) {
                     if (P.dm.d == 128)
                         reduce_qkv<128>(P, l, t, cw, lane, s, ks);
                     else
@@ -1083,7 +1087,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 bar_compute();
                 if (ct == 0) {
                     red_release_add(c, 1);
-                    if (!lt && (lin == 1 || lin == 3)) red_release_add(ctr(P, l, lin == 1 ? P.cl.res_o : P.cl.res_dn), 1);
+                    if (lin == 1 || lin == 3) red_release_add(ctr(P, l, lin == 1 ? P.cl.res_o : P.cl.res_dn), 1);
                 }
                 if (tr && ct == 0) tr[8 * i + 7] = globaltimer_ns();
             }
@@ -1212,7 +1216,6 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
         P.lora_b[i] = static_cast<const bf16 *>(L.lora_b[i]);
         P.lb_stride[i] = L.lb_stride[i];
         P.part[i] = L.part[i];
-        P.red_lora[i] = L.red_lora[i];
     }
     P.attn_norm = static_cast<const bf16 *>(L.attn_norm);
     P.mlp_norm = static_cast<const bf16 *>(L.mlp_norm);

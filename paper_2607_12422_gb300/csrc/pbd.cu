@@ -87,7 +87,7 @@ struct pbd_ctx {
     int *page_table;
     // scratch
     void *h, *q, *attn, *act, *x_ro;
-    float *part[4], *red_lora[4], *ss, *o_part;
+    float *part[4], *ss, *o_part;
     float2 *ml_part;
     float *tile_max;
     int *tile_arg;
@@ -275,7 +275,6 @@ size_t layout(pbd_ctx *c, void *base) {
     for (int lin = 0; lin < 4; ++lin) {
         c->part[lin] = (float *)bp.take(sizeof(float) * (size_t)(lin_K(k, lin) / 256) * RA *
                                         (lin_main(k, lin) + lin_lora(k, lin)));
-        c->red_lora[lin] = (float *)bp.take(sizeof(float) * (size_t)RA * lin_lora(k, lin));
     }
     c->o_part = (float *)bp.take(sizeof(float) * (size_t)RA * Hq * c->n_splits * ATT_SUBS * d);
     c->ml_part = (float2 *)bp.take(sizeof(float2) * (size_t)RA * Hq * c->n_splits * ATT_SUBS);
@@ -437,7 +436,6 @@ MKLaunch make_launch(pbd_ctx *c, const PassDesc &pd, int kind) {
         L.lora_b[lin] = c->lb[lin];
         L.lb_stride[lin] = (size_t)w0.n_main * k.lora_rank;
         L.part[lin] = c->part[lin];
-        L.red_lora[lin] = c->red_lora[lin];
     }
     L.attn_norm = c->attn_norm;
     L.mlp_norm = c->mlp_norm;

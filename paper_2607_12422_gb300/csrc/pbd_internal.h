@@ -107,7 +107,6 @@ struct MKLaunch {
     const int *ids;
     float *part[4];
     int part_rows;
-    float *red_lora[4];
     void *h, *q, *attn, *act, *x_ro;
     float *ss;
     float *o_part;
