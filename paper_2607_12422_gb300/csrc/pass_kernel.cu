@@ -186,35 +186,39 @@ __device__ __forceinline__ float row_rms(const MKParams &P, int m) {
     return __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(__fdiv_rn(a, (float)P.dm.H), P.dm.eps)));
 }
 
-// u[0..r) of row m for one adapter of linear `lin` (its rows c0 .. c0 + r - 1 in the adapter
-// tile): the bf16-rounded adapter intermediates x A^T, kept as fp32.  Summed here from the
-// adapter tile's K-slice partials (slices in order), so a main tile's reducer does not wait for
-// a separate reduction of the adapter tile.  Lane j < r sums u_j; the warp shares the vector.
-// Every lane of the warp calls it.
-__device__ __forceinline__ void lora_u(const MKParams &P, int lin, int m, int c0, int lane, float (&u)[MAX_RANK]) {
-    const int r = P.dm.r, ks = P.ks[lin];
-    const int nt = P.n_main[lin] + P.lora_rows[lin];
-    const float *p = P.part[lin] + (size_t)m * nt + P.n_main[lin] + c0 + lane;
-    const size_t stride = (size_t)P.part_rows * nt;
+// sum_j u_j * B[f, j] over j = 0..r-1 in order (B row: r bf16 values, r % 8 == 0)
+// one B row (r bf16 values) of the adapter, for lora_dot_w
+struct BRow {
+    uint4 w[MAX_RANK / 8];
+};
+__device__ __forceinline__ BRow load_brow(const bf16 *Brow, int r) {
+    BRow b;
+#pragma unroll
+    for (int q = 0; q < MAX_RANK / 8; ++q)
+        b.w[q] = q * 8 < r ? __ldg(reinterpret_cast<const uint4 *>(Brow) + q) : make_uint4(0, 0, 0, 0);
+    return b;
+}
+__device__ __forceinline__ float lora_dot_w(const float (&u)[MAX_RANK], const BRow &b, int r) {
     float a = 0.f;
-    if (lane < r) {
-        for (int s0 = 0; s0 < ks; s0 += 8) {
-            float v[8];
 #pragma unroll
-            for (int s = 0; s < 8; ++s) v[s] = s0 + s < ks ? __ldcg(p + (size_t)(s0 + s) * stride) : 0.f;
+    for (int q = 0; q < MAX_RANK / 8; ++q) {
+        if (q * 8 < r) {
+            const bf16 *e = reinterpret_cast<const bf16 *>(&b.w[q]);
 #pragma unroll
-            for (int s = 0; s < 8; ++s) {
-                if (s0 + s >= ks) break;
-                a = (s0 + s == 0) ? v[s] : __fadd_rn(a, v[s]);
-            }
+            for (int j = 0; j < 8; ++j) a = __fadd_rn(a, __fmul_rn(u[q * 8 + j], bf2f(e[j])));
         }
-        a = rbf(a);
     }
-#pragma unroll
-    for (int j = 0; j < MAX_RANK; ++j) u[j] = __shfl_sync(0xffffffffu, a, j);
+    return a;
 }
 
-// sum_j u_j * B[f, j] over j = 0..r-1 in order (B row: r bf16 values, r % 8 == 0)
+// the adapter intermediates u[0..r) of one row, from lane j's slice-ordered sum (lane j < r holds u_j
+// before rounding), shared by the warp
+__device__ __forceinline__ void share_u(float lane_sum, int base, float (&u)[MAX_RANK]) {
+    const float a = rbf(lane_sum);
+#pragma unroll
+    for (int j = 0; j < MAX_RANK; ++j) u[j] = __shfl_sync(0xffffffffu, a, base + j);
+}
+
 __device__ __forceinline__ float lora_dot_f(const float (&u)[MAX_RANK], const bf16 *Brow, int r) {
     uint4 w[MAX_RANK / 8];
 #pragma unroll
@@ -235,7 +239,7 @@ __device__ __forceinline__ float lora_dot_f(const float (&u)[MAX_RANK], const bf
 // Sums of the K-slice partials of E features of row m, slices added in order; loads go out
 // in batches of S slices (every load of a batch in flight before the first add).
 template <int E, int S>
-__device__ __forceinline__ void sum_parts(const MKParams &P, int lin, int m, const int (&f)[E], float (&out)[E]) {
+__device__ __forceinline__ void sum_parts(const MKParams &P, int lin, int m, const int *f, float *out) {
     const int nt = P.n_main[lin] + P.lora_rows[lin];
     const float *p = P.part[lin] + (size_t)m * nt;
     const size_t stride = (size_t)P.part_rows * nt;
@@ -342,7 +346,7 @@ __device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int 
 }
 
 // q|k|v tile: adapter delta, bf16, per-head RMSNorm + RoPE for q and k, store q / paged K, V
-template <int DH>
+template <int DH, bool AD>
 __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, int cw, int lane, int m0, int mstep) {
     constexpr int E = DH / 32;
     const Dims &dm = P.dm;
@@ -358,16 +362,18 @@ __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, 
         const int head = kind == 0 ? fbase / DH : (kind == 1 ? (fbase - qw) / DH : (fbase - qw - kvw) / DH);
         const int b = P.pd.b0 + m / P.pd.R;
         const int pos = P.L[b] + m % P.pd.R;
-        int f[E];
+        // features 0..E-1: the lane's outputs; feature E: the adapter row whose u lane j < r sums
+        int f[E + 1];
 #pragma unroll
         for (int j = 0; j < E; ++j) f[j] = fbase + lane + 32 * j;
+        f[E] = P.n_main[0] + kind * r + (lane < r ? lane : 0);
+        float y[E + 1];
+        sum_parts<E + (AD ? 1 : 0), 8>(P, 0, m, f, y);
         float u[MAX_RANK];
-        if (P.pd.adapter) lora_u(P, 0, m, kind * r, lane, u);
-        float y[E];
-        sum_parts<E, 8>(P, 0, m, f, y);
+        if (AD) share_u(y[E], 0, u);
 #pragma unroll
         for (int j = 0; j < E; ++j) {
-            if (P.pd.adapter) y[j] = __fadd_rn(y[j], __fmul_rn(dm.lora_scale, lora_dot_f(u, lb + (size_t)f[j] * r, r)));
+            if (AD) y[j] = __fadd_rn(y[j], __fmul_rn(dm.lora_scale, lora_dot_f(u, lb + (size_t)f[j] * r, r)));
             y[j] = rbf(y[j]);
         }
         if (kind < 2) {
@@ -414,26 +420,35 @@ __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, 
 }
 
 // o or down tile: adapter delta, residual add into h, per-tile sum of squares
+template <bool AD>
 __device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int layer, int tile, int cw, int lane, int m0,
                                              int mstep) {
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r, H = dm.H, nt = H / TILE_ROWS;
     const bf16 *lb = P.lora_b[lin] + (size_t)layer * P.lb_stride[lin];
+    if (m0 + cw * mstep >= M) return;
+    // B rows depend only on the feature: loaded once, before the rows
+    BRow br[4];
+    if (AD)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) br[e] = load_brow(lb + (size_t)(tile * TILE_ROWS + lane + 32 * e) * r, r);
     for (int m = m0 + cw * mstep; m < M; m += (CT / 32) * mstep) {
-        int f[4];
-        float hv[4], acc[4];
+        // features 0-3: the lane's outputs; feature 4: the adapter row whose u lane j < r sums
+        int f[5];
+        float hv[4], acc[5];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
             f[e] = tile * TILE_ROWS + lane + 32 * e;
             hv[e] = bf2f(ldcg_bf(P.h + (size_t)m * H + f[e]));
         }
+        f[4] = P.n_main[lin] + (lane < r ? lane : 0);
+        sum_parts<AD ? 5 : 4, 8>(P, lin, m, f, acc);
         float u[MAX_RANK];
-        if (P.pd.adapter) lora_u(P, lin, m, 0, lane, u);
-        sum_parts<4, 8>(P, lin, m, f, acc);
+        if (AD) share_u(acc[4], 0, u);
         float v[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-            if (P.pd.adapter) acc[e] = __fadd_rn(acc[e], __fmul_rn(dm.lora_scale, lora_dot_f(u, lb + (size_t)f[e] * r, r)));
+            if (AD) acc[e] = __fadd_rn(acc[e], __fmul_rn(dm.lora_scale, lora_dot_w(u, br[e], r)));
             v[e] = rbf(__fadd_rn(hv[e], rbf(acc[e])));
             P.h[(size_t)m * H + f[e]] = f2bf(v[e]);
         }
@@ -443,27 +458,38 @@ __device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int lay
 }
 
 // gate|up tile (rows 0-63 gate features 64t.., rows 64-127 up features 64t..): SiLU(gate)*up
+template <bool AD>
 __device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, int cw, int lane, int m0, int mstep) {
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r, I = dm.I;
     const bf16 *lb = P.lora_b[2] + (size_t)layer * P.lb_stride[2];
-    for (int m = m0 + cw * mstep; m < M; m += (CT / 32) * mstep) {
-        // partial rows: gate j = lane, lane+32 at tile rows j; up at tile rows 64 + j
-        const int f[4] = {tile * TILE_ROWS + lane, tile * TILE_ROWS + lane + 32, tile * TILE_ROWS + 64 + lane,
-                          tile * TILE_ROWS + 96 + lane};
-        float ug[MAX_RANK], uu[MAX_RANK], s[4];
-        if (P.pd.adapter) {
-            lora_u(P, 2, m, 0, lane, ug);
-            lora_u(P, 2, m, r, lane, uu);
+    if (m0 + cw * mstep >= M) return;
+    BRow bg[2], bu[2];
+    if (AD)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            const int a = tile * 64 + lane + 32 * e;
+            bg[e] = load_brow(lb + (size_t)a * r, r);
+            bu[e] = load_brow(lb + (size_t)(I + a) * r, r);
         }
-        sum_parts<4, 8>(P, 2, m, f, s);
+    for (int m = m0 + cw * mstep; m < M; m += (CT / 32) * mstep) {
+        // partial rows: gate j = lane, lane+32 at tile rows j; up at tile rows 64 + j; feature 4:
+        // adapter row lane (lanes 0..r-1 sum u_gate, lanes r..2r-1 u_up)
+        const int f[5] = {tile * TILE_ROWS + lane, tile * TILE_ROWS + lane + 32, tile * TILE_ROWS + 64 + lane,
+                          tile * TILE_ROWS + 96 + lane, P.n_main[2] + (lane < 2 * r ? lane : 0)};
+        float ug[MAX_RANK], uu[MAX_RANK], s[5];
+        sum_parts<AD ? 5 : 4, 2>(P, 2, m, f, s);
+        if (AD) {
+            share_u(s[4], 0, ug);
+            share_u(s[4], r, uu);
+        }
 #pragma unroll
         for (int e = 0; e < 2; ++e) {
             const int a = tile * 64 + lane + 32 * e;  // act feature
             float g = s[e], up = s[2 + e];
-            if (P.pd.adapter) {
-                g = __fadd_rn(g, __fmul_rn(dm.lora_scale, lora_dot_f(ug, lb + (size_t)a * r, r)));
-                up = __fadd_rn(up, __fmul_rn(dm.lora_scale, lora_dot_f(uu, lb + (size_t)(I + a) * r, r)));
+            if (AD) {
+                g = __fadd_rn(g, __fmul_rn(dm.lora_scale, lora_dot_w(ug, bg[e], r)));
+                up = __fadd_rn(up, __fmul_rn(dm.lora_scale, lora_dot_w(uu, bu[e], r)));
             }
             g = rbf(g);
             up = rbf(up);
@@ -1075,15 +1101,17 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 }
                 bar_compute();
                 if (!s_ok) break;
+                const bool ad = P.pd.adapter != 0;
                 if (lin == 0) {
                     if (P.dm.d == 128)
-                        reduce_qkv<128>(P, l, t, cw, lane, s, ks);
+                        ad ? reduce_qkv<128, true>(P, l, t, cw, lane, s, ks) : reduce_qkv<128, false>(P, l, t, cw, lane, s, ks);
                     else
-                        reduce_qkv<64>(P, l, t, cw, lane, s, ks);
+                        ad ? reduce_qkv<64, true>(P, l, t, cw, lane, s, ks) : reduce_qkv<64, false>(P, l, t, cw, lane, s, ks);
                 } else if (lin == 2)
-                    reduce_gu(P, l, t, cw, lane, s, ks);
+                    ad ? reduce_gu<true>(P, l, t, cw, lane, s, ks) : reduce_gu<false>(P, l, t, cw, lane, s, ks);
                 else
-                    reduce_residual(P, lin, l, t, cw, lane, s, ks);
+                    ad ? reduce_residual<true>(P, lin, l, t, cw, lane, s, ks)
+                       : reduce_residual<false>(P, lin, l, t, cw, lane, s, ks);
                 bar_compute();
                 if (ct == 0) {
                     red_release_add(c, 1);
