@@ -539,7 +539,7 @@ __device__ uint32_t attn_pages(const MKParams &P, int layer, int bl, int g, int 
 
 // One (sequence, KV head, 128-key split) on the compute group, after its K/V pages landed in
 // `smem` (stages 0 and 1 of attn_pages) and `bar` completed phase `parity`.
-template <int DH>
+template <int DH, bool BLK>
 __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, int g, int s, uint8_t *smem,
                                         uint64_t *bar, uint32_t parity, int ct, int cw, int lane,
                                         unsigned long long *stamp) {
@@ -582,7 +582,7 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
     if (stamp && ct == 0) stamp[5] = globaltimer_ns();
     if (!landed) return;
     const int gq = lane >> 2, tq = lane & 3;
-    const bool blk = P.pd.mask_mode == MASK_BLOCK_DRAFT;
+    constexpr bool blk = BLK;  // draft mask: the block's mask rows see each other
     for (int unit = cw; unit < n_mt * ATT_SUBS; unit += CT / 32) {
         const int mt = unit / ATT_SUBS, half = unit % ATT_SUBS, kb = half * HALF;
         const int qv0 = mt * 16 + gq, qv1 = qv0 + 8;
@@ -976,12 +976,14 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                         mbar_arrive_expect_tx(&att_bar, attn_pages(P, it.layer, bl, g, s, 1, uni, &att_bar, false));
                         attn_pages(P, it.layer, bl, g, s, 1, uni, &att_bar, true);
                     }
+                    unsigned long long *st = tr ? tr + 8 * i : nullptr;
+                    const bool blk = P.pd.mask_mode == MASK_BLOCK_DRAFT;
                     if (P.dm.d == 128)
-                        attn_split<128>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane,
-                                        tr ? tr + 8 * i : nullptr);
+                        blk ? attn_split<128, true>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st)
+                            : attn_split<128, false>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st);
                     else
-                        attn_split<64>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane,
-                                       tr ? tr + 8 * i : nullptr);
+                        blk ? attn_split<64, true>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st)
+                            : attn_split<64, false>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st);
                     ++ai;
                 }
                 bar_compute();
