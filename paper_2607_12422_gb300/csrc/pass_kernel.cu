@@ -812,6 +812,9 @@ __device__ bool wait_deps(const MKParams &P, const MKItem &it) {
 
 // ------------------------------------------------------------------ the kernel
 
+// DRAFT: the adapter-on pass with the block-diffusion mask; otherwise adapter off and causal.
+// One instantiation per kind keeps each kernel's code and registers to what that pass runs.
+template <bool DRAFT>
 __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ MKParams P) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -977,13 +980,10 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                         attn_pages(P, it.layer, bl, g, s, 1, uni, &att_bar, true);
                     }
                     unsigned long long *st = tr ? tr + 8 * i : nullptr;
-                    const bool blk = P.pd.mask_mode == MASK_BLOCK_DRAFT;
                     if (P.dm.d == 128)
-                        blk ? attn_split<128, true>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st)
-                            : attn_split<128, false>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st);
+                        attn_split<128, DRAFT>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st);
                     else
-                        blk ? attn_split<64, true>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st)
-                            : attn_split<64, false>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st);
+                        attn_split<64, DRAFT>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st);
                     ++ai;
                 }
                 bar_compute();
@@ -1097,23 +1097,21 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                     if (tr) tr[8 * i + 6] = globaltimer_ns();
                     bool ok = spin_until(c, ks, P);
                     // every slice of the adapter tile must be stored before a main tile adds the delta
-                    if (ok && P.pd.adapter && P.lora_rows[lin] > 0)
+                    if (ok && DRAFT && P.lora_rows[lin] > 0)
                         ok = spin_until(ctr(P, l, P.cl.lin[lin] + P.n_main[lin] / TILE_ROWS), ks, P);
                     s_ok = ok ? 1 : 0;
                 }
                 bar_compute();
                 if (!s_ok) break;
-                const bool ad = P.pd.adapter != 0;
                 if (lin == 0) {
                     if (P.dm.d == 128)
-                        ad ? reduce_qkv<128, true>(P, l, t, cw, lane, s, ks) : reduce_qkv<128, false>(P, l, t, cw, lane, s, ks);
+                        reduce_qkv<128, DRAFT>(P, l, t, cw, lane, s, ks);
                     else
-                        ad ? reduce_qkv<64, true>(P, l, t, cw, lane, s, ks) : reduce_qkv<64, false>(P, l, t, cw, lane, s, ks);
+                        reduce_qkv<64, DRAFT>(P, l, t, cw, lane, s, ks);
                 } else if (lin == 2)
-                    ad ? reduce_gu<true>(P, l, t, cw, lane, s, ks) : reduce_gu<false>(P, l, t, cw, lane, s, ks);
+                    reduce_gu<DRAFT>(P, l, t, cw, lane, s, ks);
                 else
-                    ad ? reduce_residual<true>(P, lin, l, t, cw, lane, s, ks)
-                       : reduce_residual<false>(P, lin, l, t, cw, lane, s, ks);
+                    reduce_residual<DRAFT>(P, lin, l, t, cw, lane, s, ks);
                 bar_compute();
                 if (ct == 0) {
                     red_release_add(c, 1);
@@ -1288,9 +1286,13 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
     P.union_bytes = (int)uni;
     P.b_dbl = (size_t)MAX_ATOMS * P.bn * 128 <= uni ? 1 : 0;
     const size_t dyn = (size_t)P.ring_bytes + uni + 1024;
+    // the two pass kinds the kernel is built for
+    const bool draft = L.pd.adapter != 0;
+    if (draft != (L.pd.mask_mode == MASK_BLOCK_DRAFT)) return cudaErrorInvalidValue;
     static size_t configured = 0;
     if (dyn > configured) {
-        e = cudaFuncSetAttribute(k_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+        e = cudaFuncSetAttribute(k_pass<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+        if (e == cudaSuccess) e = cudaFuncSetAttribute(k_pass<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
         if (e != cudaSuccess) return e;
         configured = dyn;
     }
@@ -1304,7 +1306,7 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
     attr[0].val.cooperative = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, k_pass, P);
+    return draft ? cudaLaunchKernelEx(&cfg, k_pass<true>, P) : cudaLaunchKernelEx(&cfg, k_pass<false>, P);
 }
 
 }  // namespace pbd
