@@ -814,7 +814,7 @@ __device__ bool wait_deps(const MKParams &P, const MKItem &it) {
 
 // DRAFT: the adapter-on pass with the block-diffusion mask; otherwise adapter off and causal.
 // One instantiation per kind keeps each kernel's code and registers to what that pass runs.
-template <bool DRAFT>
+template <bool DRAFT, int DH>
 __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ MKParams P) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -980,10 +980,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                         attn_pages(P, it.layer, bl, g, s, 1, uni, &att_bar, true);
                     }
                     unsigned long long *st = tr ? tr + 8 * i : nullptr;
-                    if (P.dm.d == 128)
-                        attn_split<128, DRAFT>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st);
-                    else
-                        attn_split<64, DRAFT>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st);
+                    attn_split<DH, DRAFT>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st);
                     ++ai;
                 }
                 bar_compute();
@@ -1008,10 +1005,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 if (!s_ok) break;
                 if (s_red) {
                     const int p0 = shared_merge ? s : 0, pstep = shared_merge ? nsp : 1;
-                    if (P.dm.d == 128)
-                        attn_combine<128>(P, bl, g, cw, lane, p0, pstep);
-                    else
-                        attn_combine<64>(P, bl, g, cw, lane, p0, pstep);
+                    attn_combine<DH>(P, bl, g, cw, lane, p0, pstep);
                     bar_compute();
                     if (ct == 0) red_release_add(c, 1);
                     if (tr && ct == 0) tr[8 * i + 7] = globaltimer_ns();
@@ -1104,10 +1098,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 bar_compute();
                 if (!s_ok) break;
                 if (lin == 0) {
-                    if (P.dm.d == 128)
-                        reduce_qkv<128, DRAFT>(P, l, t, cw, lane, s, ks);
-                    else
-                        reduce_qkv<64, DRAFT>(P, l, t, cw, lane, s, ks);
+                    reduce_qkv<DH, DRAFT>(P, l, t, cw, lane, s, ks);
                 } else if (lin == 2)
                     reduce_gu<DRAFT>(P, l, t, cw, lane, s, ks);
                 else
@@ -1291,8 +1282,10 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
     if (draft != (L.pd.mask_mode == MASK_BLOCK_DRAFT)) return cudaErrorInvalidValue;
     static size_t configured = 0;
     if (dyn > configured) {
-        e = cudaFuncSetAttribute(k_pass<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
-        if (e == cudaSuccess) e = cudaFuncSetAttribute(k_pass<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+        e = cudaFuncSetAttribute(k_pass<true, 128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+        if (e == cudaSuccess) e = cudaFuncSetAttribute(k_pass<false, 128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+        if (e == cudaSuccess) e = cudaFuncSetAttribute(k_pass<true, 64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+        if (e == cudaSuccess) e = cudaFuncSetAttribute(k_pass<false, 64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
         if (e != cudaSuccess) return e;
         configured = dyn;
     }
@@ -1306,7 +1299,9 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
     attr[0].val.cooperative = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return draft ? cudaLaunchKernelEx(&cfg, k_pass<true>, P) : cudaLaunchKernelEx(&cfg, k_pass<false>, P);
+    if (L.dm.d == 128)
+        return draft ? cudaLaunchKernelEx(&cfg, k_pass<true, 128>, P) : cudaLaunchKernelEx(&cfg, k_pass<false, 128>, P);
+    return draft ? cudaLaunchKernelEx(&cfg, k_pass<true, 64>, P) : cudaLaunchKernelEx(&cfg, k_pass<false, 64>, P);
 }
 
 }  // namespace pbd
