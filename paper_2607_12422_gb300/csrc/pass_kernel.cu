@@ -973,11 +973,12 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 const int bl = it.a, g = it.b, s = it.c;
                 if (att_active) {
                     if (ct == 0) {
+                        const uint32_t nb1 = attn_pages(P, it.layer, bl, g, s, 1, uni, &att_bar, false);
                         // the block's pages were written by this pass's q|k|v reducers (generic
                         // stores, acquired above); order them before the TMA reads
-                        fence_proxy_async_global();
-                        mbar_arrive_expect_tx(&att_bar, attn_pages(P, it.layer, bl, g, s, 1, uni, &att_bar, false));
-                        attn_pages(P, it.layer, bl, g, s, 1, uni, &att_bar, true);
+                        if (nb1) fence_proxy_async_global();
+                        mbar_arrive_expect_tx(&att_bar, nb1);
+                        if (nb1) attn_pages(P, it.layer, bl, g, s, 1, uni, &att_bar, true);
                     }
                     unsigned long long *st = tr ? tr + 8 * i : nullptr;
                     attn_split<DH, DRAFT>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st);
