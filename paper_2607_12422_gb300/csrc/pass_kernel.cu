@@ -604,14 +604,19 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
             sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
-            const int n = kb + nt * 8 + gq;
+            // K fragments of two k-steps per ldmatrix.x4: matrix j = keys n0..n0+7, dims 8j..8j+7
+            // of the 32-dim chunk; thread t addresses row t % 8 of matrix t / 8
+            const int kr = kb + nt * 8 + (lane & 7);
 #pragma unroll
-            for (int ks = 0; ks < KS; ++ks) {
-                const int e = ks * 16 + 2 * tq;
-                const uint8_t *kb = sK + (e >> 6) * ATT_SUB_BYTES;
-                const uint32_t b0 = *reinterpret_cast<const uint32_t *>(kb + sw128(n, (e & 63) * 2));
-                const uint32_t b1 = *reinterpret_cast<const uint32_t *>(kb + sw128(n, ((e + 8) & 63) * 2));
+            for (int ks = 0; ks < KS; ks += 2) {
+                const int e = ks * 16 + (lane >> 3) * 8;
+                const uint32_t addr = smem_u32(sK + (e >> 6) * ATT_SUB_BYTES + sw128(kr, (e & 63) * 2));
+                uint32_t b0, b1, b2, b3;
+                asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                             : "=r"(b0), "=r"(b1), "=r"(b2), "=r"(b3)
+                             : "r"(addr));
                 mma_m16n8k16_bf16(sc[nt], qa[ks], b0, b1);
+                mma_m16n8k16_bf16(sc[nt], qa[ks + 1], b2, b3);
             }
         }
         const int qp0 = L + i0, qp1 = L + i1;
