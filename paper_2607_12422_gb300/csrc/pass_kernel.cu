@@ -721,34 +721,42 @@ __device__ __noinline__ void attn_combine(const MKParams &P, int bl, int g, int 
         const int m = bl * R + i;
         const float2 *ml = P.ml_part + ((size_t)m * dm.Hq + h) * nsa;
         const float *ob = P.o_part + ((size_t)m * dm.Hq + h) * nsa * DH + lane;
+        // the first 16 partial results' statistics and the first 8 outputs go out together
+        constexpr int NB = 16, OB = 8;
+        float2 v[NB];
+        float o[OB][E];
+#pragma unroll
+        for (int u = 0; u < NB; ++u) v[u] = u < nv ? __ldcg(ml + u) : make_float2(-INFINITY, 0.f);
+#pragma unroll
+        for (int u = 0; u < OB; ++u)
+#pragma unroll
+            for (int e = 0; e < E; ++e) o[u][e] = u < nv ? __ldcg(ob + (size_t)u * DH + 32 * e) : 0.f;
         float mx = -INFINITY;
-        for (int s0 = 0; s0 < nv; s0 += 8) {
-            float2 v[8];
 #pragma unroll
-            for (int u = 0; u < 8; ++u) v[u] = s0 + u < nv ? __ldcg(ml + s0 + u) : make_float2(-INFINITY, 0.f);
-#pragma unroll
-            for (int u = 0; u < 8; ++u)
-                if (v[u].y > 0.f) mx = fmaxf(mx, v[u].x);
+        for (int u = 0; u < NB; ++u)
+            if (v[u].y > 0.f) mx = fmaxf(mx, v[u].x);
+        for (int s0 = NB; s0 < nv; ++s0) {  // long contexts only
+            const float2 w = __ldcg(ml + s0);
+            if (w.y > 0.f) mx = fmaxf(mx, w.x);
         }
         float num[E];
 #pragma unroll
         for (int e = 0; e < E; ++e) num[e] = 0.f;
         float den = 0.f;
-        for (int s0 = 0; s0 < nv; s0 += 4) {
-            float2 v[4];
-            float o[4][E];
+        for (int s0 = 0; s0 < nv; s0 += OB) {
+            if (s0 > 0)
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const bool in = s0 + u < nv;
-                v[u] = in ? __ldcg(ml + s0 + u) : make_float2(-INFINITY, 0.f);
+                for (int u = 0; u < OB; ++u)
 #pragma unroll
-                for (int e = 0; e < E; ++e) o[u][e] = in ? __ldcg(ob + (size_t)(s0 + u) * DH + 32 * e) : 0.f;
-            }
+                    for (int e = 0; e < E; ++e) o[u][e] = s0 + u < nv ? __ldcg(ob + (size_t)(s0 + u) * DH + 32 * e) : 0.f;
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                if (!(v[u].y > 0.f)) continue;  // the row saw no key in this split
-                const float w = __expf(v[u].x - mx);
-                den = __fadd_rn(den, __fmul_rn(w, v[u].y));
+            for (int u = 0; u < OB; ++u) {
+                const int sp = s0 + u;
+                if (sp >= nv) break;
+                const float2 st = sp < NB ? v[sp < NB ? sp : 0] : __ldcg(ml + sp);
+                if (!(st.y > 0.f)) continue;  // the row saw no key in this partial result
+                const float w = __expf(st.x - mx);
+                den = __fadd_rn(den, __fmul_rn(w, st.y));
 #pragma unroll
                 for (int e = 0; e < E; ++e) num[e] = __fadd_rn(num[e], __fmul_rn(w, o[u][e]));
             }
