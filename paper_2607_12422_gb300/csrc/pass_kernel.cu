@@ -620,6 +620,10 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
             }
         }
         const int qp0 = L + i0, qp1 = L + i1;
+        // last visible key of each row: causal rows see up to themselves; in the draft the
+        // block's mask rows (i >= 1) also see the rest of the block
+        const int lim0 = val0 ? ((blk && i0 >= 1) ? T - 1 : qp0) : -1;
+        const int lim1 = val1 ? ((blk && i1 >= 1) ? T - 1 : qp1) : -1;
         const float scale = P.att_scale;
         float m0 = -INFINITY, m1 = -INFINITY;
 #pragma unroll
@@ -627,8 +631,8 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
                 const int kp = k0 + kb + nt * 8 + 2 * tq + e;
-                const bool vis0 = val0 && kp < T && (kp <= qp0 || (blk && i0 >= 1 && kp > L));
-                const bool vis1 = val1 && kp < T && (kp <= qp1 || (blk && i1 >= 1 && kp > L));
+                const bool vis0 = kp <= lim0;
+                const bool vis1 = kp <= lim1;
                 sc[nt][e] = vis0 ? __fmul_rn(sc[nt][e], scale) : -INFINITY;
                 sc[nt][2 + e] = vis1 ? __fmul_rn(sc[nt][2 + e], scale) : -INFINITY;
                 m0 = fmaxf(m0, sc[nt][e]);
