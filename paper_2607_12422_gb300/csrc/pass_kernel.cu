@@ -127,6 +127,23 @@ __device__ bool spin_until(const int *c, int target, const MKParams &P) {
     }
 }
 
+// one thread: wait until *c1 >= t1 and *c2 >= t2, both polled in each round (bounded)
+__device__ bool spin_until2(const int *c1, int t1, const int *c2, int t2, const MKParams &P) {
+    const uint64_t t0 = globaltimer_ns();
+    for (;;) {
+        for (int i = 0; i < 8; ++i) {
+            const int v1 = ld_acquire(c1), v2 = ld_acquire(c2);
+            if (v1 >= t1 && v2 >= t2) return true;
+            __nanosleep(40);
+        }
+        if (aborted(P)) return false;
+        if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
+            raise_abort(P, DEV_TIMEOUT_DEP);
+            return false;
+        }
+    }
+}
+
 // bounded mbarrier wait that also gives up when the pass is aborted
 __device__ bool mbar_wait_mk(uint64_t *bar, uint32_t parity, const MKParams &P, int code) {
     const uint32_t a = smem_u32(bar);
@@ -1107,10 +1124,11 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 if (ct == 0) {
                     red_release_add(c, 1);
                     if (tr) tr[8 * i + 6] = globaltimer_ns();
-                    bool ok = spin_until(c, ks, P);
-                    // every slice of the adapter tile must be stored before a main tile adds the delta
-                    if (ok && DRAFT && P.lora_rows[lin] > 0)
-                        ok = spin_until(ctr(P, l, P.cl.lin[lin] + P.n_main[lin] / TILE_ROWS), ks, P);
+                    // with the adapter, every slice of the adapter tile must be stored too (both
+                    // counters polled together)
+                    const bool ok = (DRAFT && P.lora_rows[lin] > 0)
+                                        ? spin_until2(c, ks, ctr(P, l, P.cl.lin[lin] + P.n_main[lin] / TILE_ROWS), ks, P)
+                                        : spin_until(c, ks, P);
                     s_ok = ok ? 1 : 0;
                 }
                 bar_compute();
