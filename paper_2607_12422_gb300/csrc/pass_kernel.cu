@@ -236,23 +236,6 @@ __device__ __forceinline__ void share_u(float lane_sum, int base, float (&u)[MAX
     for (int j = 0; j < MAX_RANK; ++j) u[j] = __shfl_sync(0xffffffffu, a, base + j);
 }
 
-__device__ __forceinline__ float lora_dot_f(const float (&u)[MAX_RANK], const bf16 *Brow, int r) {
-    uint4 w[MAX_RANK / 8];
-#pragma unroll
-    for (int q = 0; q < MAX_RANK / 8; ++q)
-        if (q * 8 < r) w[q] = __ldg(reinterpret_cast<const uint4 *>(Brow) + q);
-    float a = 0.f;
-#pragma unroll
-    for (int q = 0; q < MAX_RANK / 8; ++q) {
-        if (q * 8 < r) {
-            const bf16 *e = reinterpret_cast<const bf16 *>(&w[q]);
-#pragma unroll
-            for (int j = 0; j < 8; ++j) a = __fadd_rn(a, __fmul_rn(u[q * 8 + j], bf2f(e[j])));
-        }
-    }
-    return a;
-}
-
 // Sums of the K-slice partials of E features of row m, slices added in order; loads go out
 // in batches of S slices (every load of a batch in flight before the first add).
 template <int E, int S>
@@ -384,13 +367,17 @@ __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, 
 #pragma unroll
         for (int j = 0; j < E; ++j) f[j] = fbase + lane + 32 * j;
         f[E] = P.n_main[0] + kind * r + (lane < r ? lane : 0);
+        BRow br[E];  // the lane's B rows, in flight with the partial sums
+        if (AD)
+#pragma unroll
+            for (int j = 0; j < E; ++j) br[j] = load_brow(lb + (size_t)f[j] * r, r);
         float y[E + 1];
         sum_parts<E + (AD ? 1 : 0), 8>(P, 0, m, f, y);
         float u[MAX_RANK];
         if (AD) share_u(y[E], 0, u);
 #pragma unroll
         for (int j = 0; j < E; ++j) {
-            if (AD) y[j] = __fadd_rn(y[j], __fmul_rn(dm.lora_scale, lora_dot_f(u, lb + (size_t)f[j] * r, r)));
+            if (AD) y[j] = __fadd_rn(y[j], __fmul_rn(dm.lora_scale, lora_dot_w(u, br[j], r)));
             y[j] = rbf(y[j]);
         }
         if (kind < 2) {
