@@ -198,3 +198,28 @@ def test_state_machine_errors(env):
     with pytest.raises(pbd.PbdError) as ei:
         eng.pbd_prefill([np.zeros(300, np.int32)], max_new=8)
     assert ei.value.status == 3
+
+
+def test_pass_timing_and_trace_entry_points(env):
+    """pbd_time_pass and pbd_trace_pass run a pass on a prefilled context without advancing it:
+    positive times and byte counts, every scheduled item traced once with ordered stamps, and
+    the generation state unchanged afterwards."""
+    eng, prompt = env["eng"], env["prompts"][1]
+    eng.pbd_prefill([prompt], max_new=32)
+    before = [np.asarray(x).copy() for x in eng.pbd_get_state()]
+    for kind in (0, 1, 2):
+        ms, nbytes = eng.pbd_time_pass(kind, 2)
+        assert ms > 0 and nbytes > 0
+        items, st = eng.pbd_trace_pass(kind)
+        assert len(items) == len(st) > 0
+        assert st.shape[1] == 8
+        ops = items[:, 0] & 0xFF
+        assert set(np.unique(ops)) <= {0, 1, 2, 3}
+        # start <= inputs ready <= end for every item (all stamps from one global clock)
+        assert (st[:, 0] > 0).all() and (st[:, 1] >= st[:, 0]).all() and (st[:, 3] >= st[:, 1]).all()
+    after = [np.asarray(x) for x in eng.pbd_get_state()]
+    for a, b in zip(before, after):
+        assert np.array_equal(a, b)
+    # the context is still in the state a round starts from
+    d1, _ = eng.pbd_draft_block()
+    assert d1.shape == (1, D)
