@@ -5,6 +5,7 @@ may import this package.  The GPU product path never imports, links or runs it, 
 it imports nothing from the GPU package: it takes plain numpy arrays (bf16 bit
 patterns as uint16) and computes what the paper defines.
 """
-from .model import (OracleModel, OracleCache, accept_length, greedy_generate, spec_generate,  # noqa: F401
-                    adapter_param_count, base_param_count, MASK_CAUSAL, MASK_BLOCK_DRAFT)
+from .model import (OracleModel, OracleCache, accept_length, draft_block, greedy_generate,  # noqa: F401
+                    spec_generate, adapter_param_count, base_param_count, MASK_CAUSAL, MASK_BLOCK_DRAFT,
+                    LINEAR_NAMES)
 from .report import draft_cost_table, break_even_accept, predicted_tokens_per_s  # noqa: F401

@@ -181,11 +181,19 @@ class OracleModel:
 
     def forward(self, cache: OracleCache, L: int, tokens: Sequence[int], adapter_on: bool, mask_mode: int,
                 read_first: int = 0, n_read: Optional[int] = None, want_logits: bool = False,
-                want_hidden: bool = False):
+                want_hidden: bool = False, n_layers: Optional[int] = None):
         """One pass over len(tokens) rows at positions L.. (token < 0 = mask row).
 
+        n_layers: run only the first n_layers decoder layers, then the final norm and the tied
+        head (the early exit of Section 6); the skipped layers' cache slots are left untouched.
         Returns (argmax[n_read], logits[n_read, V] or None, hidden[n_read, H] or None).
         """
+        cfg = self.cfg
+        if n_layers is not None:
+            if not 1 <= n_layers <= self.shape.n_layers:
+                raise ValueError("n_layers %d outside [1, %d]" % (n_layers, self.shape.n_layers))
+            cfg = _Config.from_buffer_copy(self.cfg)
+            cfg.n_layers = n_layers
         toks = np.ascontiguousarray(np.asarray(tokens, dtype=np.int32))
         n = toks.shape[0]
         if n_read is None:
@@ -193,7 +201,7 @@ class OracleModel:
         am = np.empty(n_read, dtype=np.int32)
         logits = np.empty((n_read, self.shape.vocab), dtype=np.float32) if want_logits else None
         hidden = np.empty((n_read, self.shape.hidden), dtype=np.float32) if want_hidden else None
-        rc = lib(self.acc).orc_forward(C.byref(self.cfg), C.byref(self.weights), cache.ptr, L, n, _i32(toks),
+        rc = lib(self.acc).orc_forward(C.byref(cfg), C.byref(self.weights), cache.ptr, L, n, _i32(toks),
                                int(adapter_on), mask_mode, read_first, n_read,
                                _fp(logits) if logits is not None else None, _i32(am),
                                _fp(hidden) if hidden is not None else None)
@@ -224,6 +232,35 @@ def accept_length(draft: Sequence[int], verify: Sequence[int]) -> int:
     return n
 
 
+def draft_block(model: OracleModel, cache: OracleCache, L: int, p: int, D: int, draft_layers: Optional[int] = None,
+                denoise_steps: int = 1, anchored: bool = True, want_logits: bool = False):
+    """The adapter-on draft of one round (Section 3, steps 1-2) and its variants.
+
+    Step 1 runs rows [p, MASK x D] at positions L..L+D under the block mask.  The token it
+    proposes for position L+j (j = 1..D) is d_j:
+      anchored (the default): row j-1 proposes position L+j (rows 0..D-1 are read);
+      unanchored (ablation of Sections 4.4 and 5.3): mask row j proposes its own position
+        (rows 1..D are read; the pending token's row is context only).
+    denoise_steps > 1 (the two-step ablation of Sections 4.4 and 5.3): each further step
+    runs the same adapter-on block pass with the mask rows replaced by the previous step's
+    proposals, rows [p, d_1..d_D], nothing remasked; its proposals replace the block.
+    draft_layers: the draft exits after the first draft_layers decoder layers (the early exit
+    Section 6 names as a cheaper draft path); None runs all of them.
+    Returns (drafts of the last step, its logits or None, proposals of every step).
+    """
+    first = 0 if anchored else 1
+    rows = [p] + [-1] * D
+    steps = []
+    lg = None
+    for _ in range(max(1, denoise_steps)):
+        am, lg, _ = model.forward(cache, L, rows, True, MASK_BLOCK_DRAFT, first, D, want_logits=want_logits,
+                                  n_layers=draft_layers)
+        drafts = [int(t) for t in am]
+        steps.append(drafts)
+        rows = [p] + drafts
+    return steps[-1], lg, steps
+
+
 def greedy_generate(model: OracleModel, prompt: Sequence[int], max_new: int):
     """Plain greedy decoding by the adapter-off verifier: the output exact verification must reproduce."""
     P = len(prompt)
@@ -240,13 +277,15 @@ def greedy_generate(model: OracleModel, prompt: Sequence[int], max_new: int):
 def spec_generate(model: OracleModel, prompt: Sequence[int], max_new: int, D: int,
                   forced_n: Optional[Sequence[int]] = None,
                   draft_override: Optional[Callable[[int, List[int]], List[int]]] = None,
-                  want_logits: bool = False, max_rounds: Optional[int] = None, return_state: bool = False):
+                  want_logits: bool = False, max_rounds: Optional[int] = None, return_state: bool = False,
+                  draft_layers: Optional[int] = None, denoise_steps: int = 1, anchored: bool = True):
     """PEFT-BD decoding (Section 3).  Returns (tokens, rounds[, (cache, L)]).
 
     rounds[i] = dict(L=cached length before the round, pending, draft, verify, n, emitted,
-    [draft_logits, verify_logits]).  forced_n replaces the accepted length of round i by
-    forced_n[i] (timing mode); draft_override(i, drafts) may replace the drafted block
-    (adversarial drafters in the tests).  The generation budget is the only stop rule:
+    draft_steps, [draft_logits, verify_logits]).  forced_n replaces the accepted length of
+    round i by forced_n[i] (timing mode); draft_override(i, drafts) may replace the drafted
+    block (adversarial drafters in the tests).  draft_layers, denoise_steps and anchored
+    select the draft variant (draft_block).  The generation budget is the only stop rule:
     the last round is truncated to max_new tokens.
     """
     P = len(prompt)
@@ -256,9 +295,8 @@ def spec_generate(model: OracleModel, prompt: Sequence[int], max_new: int, D: in
     rounds = []
     while len(out) < max_new and (max_rounds is None or len(rounds) < max_rounds):
         ri = len(rounds)
-        d_am, d_lg, _ = model.forward(cache, L, [p] + [-1] * D, True, MASK_BLOCK_DRAFT, 0, D,
-                                      want_logits=want_logits)
-        drafts = [int(t) for t in d_am]
+        drafts, d_lg, d_steps = draft_block(model, cache, L, p, D, draft_layers, denoise_steps, anchored,
+                                            want_logits)
         if draft_override is not None:
             drafts = [int(t) for t in draft_override(ri, list(drafts))]
         v_am, v_lg, _ = model.forward(cache, L, [p] + drafts, False, MASK_CAUSAL, 0, D + 1,
@@ -269,7 +307,7 @@ def spec_generate(model: OracleModel, prompt: Sequence[int], max_new: int, D: in
             n = int(forced_n[ri])
         emitted = drafts[:n] + [verify[n]]
         take = min(len(emitted), max_new - len(out))
-        rec = dict(L=L, pending=p, draft=drafts, verify=verify, n=n, emitted=emitted[:take])
+        rec = dict(L=L, pending=p, draft=drafts, verify=verify, n=n, emitted=emitted[:take], draft_steps=d_steps)
         if want_logits:
             rec["draft_logits"], rec["verify_logits"] = d_lg, v_lg
         rounds.append(rec)
