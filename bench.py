@@ -32,6 +32,10 @@ if ROOT not in sys.path:
 WORKLOAD = "qwen3-0.6b-b1-d16-p512-g256"
 METRIC = "decoded tokens/s (PEFT-BD draft+verify rounds, Qwen3-0.6B shape, D=16)"
 CHUNK = 32  # rounds per timed chunk
+# draft variants measured beside the method of Section 3: early exit at half and quarter depth
+# (Section 6), two-step denoising and the unanchored readout (Sections 4.4 and 5.3)
+VARIANTS = (("early_exit_14", dict(draft_layers=14)), ("early_exit_7", dict(draft_layers=7)),
+            ("denoise_2", dict(denoise_steps=2)), ("unanchored", dict(anchored=False)))
 
 
 def peaks():
@@ -221,32 +225,34 @@ def main(args):
     P, G = len(prompt), Wl.max_new
     eng = pbd.Engine(S, base, ad, block_D=D, max_batch=1, max_seq_len=P + G + 8, device=dev)
 
-    def timed_rounds(mode, steps, warmup, forced=None):
-        """`warmup` then `steps` timed rounds over generations of the workload.  A chunk never holds
+    def timed_rounds(mode, steps, warmup, forced=None, e=None):
+        """`warmup` then `steps` timed rounds over generations of the workload (on engine e,
+        default the main one).  A chunk never holds
         more rounds than the budget left could absorb at full acceptance, so no timed round runs
         past a finished generation; a new prompt is prefilled (untimed) when the budget is spent.
         Returns (per-phase ms sums, tokens emitted in timed rounds, kernel launches, mean L)."""
+        e = e or eng
         acc = np.zeros(4)
         tokens = 0
         launches = 0
         l_sum = 0.0
         per_round = (D + 1) if mode == 0 else 1
-        eng.pbd_prefill([prompt], max_new=G)
+        e.pbd_prefill([prompt], max_new=G)
         done_w, left = 0, steps
         while done_w < warmup or left > 0:
-            L0, _, n0 = eng.pbd_get_state()
+            L0, _, n0 = e.pbd_get_state()
             room = (G - int(n0[0])) // per_round
             if room < 1:
-                eng.pbd_prefill([prompt], max_new=G)
+                e.pbd_prefill([prompt], max_new=G)
                 continue
             if done_w < warmup:
                 k = min(warmup - done_w, room, CHUNK)
-                eng.pbd_bench_rounds(mode, 0, k, forced)
+                e.pbd_bench_rounds(mode, 0, k, forced)
                 done_w += k
                 continue
             k = min(left, room, CHUNK)
-            r = eng.pbd_bench_rounds(mode, 0, k, forced)
-            L1, _, n1 = eng.pbd_get_state()
+            r = e.pbd_bench_rounds(mode, 0, k, forced)
+            L1, _, n1 = e.pbd_get_state()
             acc += np.array(r[:4])
             tokens += int(n1[0]) - int(n0[0])
             launches += r[4] * k
@@ -318,6 +324,27 @@ def main(args):
             e2e_vals.append(G / dt)
     e2e = float(np.median(e2e_vals))
 
+    # ---- draft variants (Sections 4.4, 5.3 and 6): same workload, natural acceptance, one
+    # engine each; the draft time covers every denoising pass and its lm_head
+    variants = None
+    if ws == 1 and not args.no_variants:
+        variants = {}
+        for name, kw in VARIANTS:
+            ev = pbd.Engine(S, base, ad, block_D=D, max_batch=1, max_seq_len=P + G + 8, device=dev, **kw)
+            v_steps = 64
+            acc_v, tok_v, _, L_v = timed_rounds(0, v_steps, args.warmup, e=ev)
+            ev.pbd_prefill([prompt], max_new=G)
+            ms_vd, vd_bytes = ev.pbd_time_pass(0, 8)
+            d_us, v_us = 1e3 * acc_v[0] / v_steps, 1e3 * acc_v[1] / v_steps
+            variants[name] = {"config": kw, "draft_us": d_us, "verify_us": v_us,
+                              "mean_tokens_per_round": tok_v / v_steps,
+                              "tokens_per_s": tok_v / (acc_v[3] / 1e3), "draft_over_verify": d_us / v_us,
+                              "draft_pass_kernel_us": ms_vd * 1e3,
+                              "draft_pass_kernel_frac": vd_bytes / (ms_vd * 1e-3) / 1e9 / hbm,
+                              "break_even_accept": (d_us + v_us) / ar_us, "steps": v_steps}
+            ev.close()
+            del ev
+
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         tps, sec, done, threads = run_cpu_oracle(S, base, ad, 64, D, 24, max_seconds=20)
@@ -341,6 +368,7 @@ def main(args):
                        "mean_tokens_per_round": mean_A, "draft_over_verify": draft_us / verify_us},
             "ar": {"us_per_step": ar_us, "pass_us": ar_pass_us, "tokens_per_s": tok_ar / (acc_ar[3] / 1e3),
                    "break_even_accept": (draft_us + verify_us) / ar_us},
+            "draft_variants": variants,
             "roofline": {"bound": "hbm", "kernel": "k_pass (persistent; 28 layers of one verify pass, 17 rows)",
                          "achieved": achieved, "peak": hbm, "peak_kind": peak_kind + " hbm_gbs (burst)",
                          "unit": "GB/s", "frac": achieved / hbm, "traffic": traffic,
@@ -369,6 +397,7 @@ if __name__ == "__main__":
     ap.add_argument("--warmup", type=int, default=8)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-variants", action="store_true", help="skip the draft-variant measurements")
     ap.add_argument("--profile-rounds", action="store_true",
                     help="only prefill + warm-up + timed rounds (the configuration profiled under ncu)")
     a = ap.parse_args()

@@ -59,6 +59,16 @@ typedef struct {
     int32_t max_batch;  /* sequences decoded together */
     int32_t max_seq_len;/* prompt + generated tokens per sequence (the D+1 scratch slots are added internally) */
     int32_t page_size;  /* KV page length in tokens; must be 16 */
+    /* Draft variants; all zero = the method of Section 3 (one adapter-on pass over every layer,
+     * row j-1 proposing position L+j).  Fixed for the context's lifetime. */
+    int32_t draft_layers;     /* early exit (Section 6): the draft runs only the first draft_layers
+                                 decoder layers before the final norm and the head; 0 = all */
+    int32_t denoise_steps;    /* adapter-on block passes per draft (the two-step ablation of Sections
+                                 4.4 and 5.3): each pass after the first refills the mask rows with the
+                                 previous pass's proposals; 0 or 1 = one pass, at most 8 */
+    int32_t draft_unanchored; /* 1: mask row j proposes its own position L+j (rows 1..D are read, the
+                                 pending token's row is context only; the unanchored ablation of
+                                 Sections 4.4 and 5.3); 0: row j-1 proposes position L+j */
 } pbd_config;
 
 /* Backbone weights: bf16, row-major [out, in] per linear, stacked over layers.  They are

@@ -827,7 +827,7 @@ __device__ bool wait_deps(const MKParams &P, const MKItem &it) {
                wait_tiles(P, l, 0, qw + g * d, qw + (g + 1) * d) &&
                wait_tiles(P, l, 0, qw + kvw + g * d, qw + kvw + (g + 1) * d);
     }
-    if (it.op == MK_FINAL) return spin_until(ctr(P, dm.nl - 1, P.cl.res_dn), dm.H / TILE_ROWS * P.ks[3], P);
+    if (it.op == MK_FINAL) return spin_until(ctr(P, P.pd.nl_run - 1, P.cl.res_dn), dm.H / TILE_ROWS * P.ks[3], P);
     return true;
 }
 
@@ -1202,7 +1202,7 @@ void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int
         for (int t = 0; t < n_main[lin]; ++t)
             for (int s = 0; s < ks; ++s) push(MK_LINEAR, lin, l, t, s, 0);
     };
-    for (int l = 0; l < dm.nl; ++l) {
+    for (int l = 0; l < pd.nl_run; ++l) {
         linear(0, l);
         for (int bl = 0; bl < pd.nb; ++bl)
             for (int g = 0; g < dm.Hkv; ++g)
@@ -1213,7 +1213,7 @@ void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int
     }
     for (int bl = 0; bl < pd.nb; ++bl)
         for (int i = pd.ro_first; i < pd.ro_first + pd.ro_count; ++i)
-            push(MK_FINAL, 0, dm.nl - 1, bl * pd.ro_count + (i - pd.ro_first), bl * pd.R + i, 0);
+            push(MK_FINAL, 0, pd.nl_run - 1, bl * pd.ro_count + (i - pd.ro_first), bl * pd.R + i, 0);
     off->assign(grid + 1, 0);
     for (size_t i = 0; i < all.size(); ++i) (*off)[i % grid + 1]++;
     for (int c = 0; c < grid; ++c) (*off)[c + 1] += (*off)[c];
@@ -1240,6 +1240,7 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
     P.vmap = *L.vmap;
     P.dm = L.dm;
     P.pd = L.pd;
+    if (L.pd.nl_run < 1 || L.pd.nl_run > L.dm.nl) return cudaErrorInvalidValue;
     P.items = L.items;
     P.cta_off = L.cta_off;
     P.cnt = L.cnt;

@@ -173,6 +173,9 @@ bool valid_config(const pbd_config *cfg, std::string *why) {
     if (k.max_batch * (k.block_D + 1) > 256) return bad("max_batch * (block_D + 1) must be <= 256");
     if (k.max_seq_len < 2 || k.max_seq_len > (1 << 20)) return bad("max_seq_len out of range");
     if (!(k.rms_eps > 0.f) || !(k.rope_theta > 0.f)) return bad("rms_eps and rope_theta must be positive");
+    if (k.draft_layers < 0 || k.draft_layers > k.n_layers) return bad("draft_layers must be in [0, n_layers]");
+    if (k.denoise_steps < 0 || k.denoise_steps > 8) return bad("denoise_steps must be in [0, 8]");
+    if (k.draft_unanchored != 0 && k.draft_unanchored != 1) return bad("draft_unanchored must be 0 or 1");
     return true;
 }
 
@@ -380,6 +383,11 @@ pbd_status build_rope(pbd_ctx *c) {
     return PBD_OK;
 }
 
+// decoder layers a pass of this kind runs: the draft may exit early, every other pass runs all
+int draft_pass_layers(const pbd_ctx *c, int kind) {
+    return (kind == PK_DRAFT && c->cfg.draft_layers > 0) ? c->cfg.draft_layers : c->cfg.n_layers;
+}
+
 PassDesc block_pass(pbd_ctx *c, int kind) {
     PassDesc pd;
     pd.b0 = 0;
@@ -388,8 +396,11 @@ PassDesc block_pass(pbd_ctx *c, int kind) {
     pd.M = pd.nb * pd.R;
     pd.adapter = kind == PK_DRAFT ? 1 : 0;
     pd.mask_mode = kind == PK_DRAFT ? MASK_BLOCK_DRAFT : MASK_CAUSAL;
-    pd.ro_first = 0;
+    // the draft reads D rows: rows 0..D-1 (row j-1 proposes position L+j) or, unanchored,
+    // the mask rows 1..D (each proposes its own position)
+    pd.ro_first = (kind == PK_DRAFT && c->cfg.draft_unanchored) ? 1 : 0;
     pd.ro_count = kind == PK_DRAFT ? c->D : pd.R;
+    pd.nl_run = draft_pass_layers(c, kind);
     return pd;
 }
 
@@ -490,8 +501,14 @@ pbd_status run_pass(pbd_ctx *c, const PassDesc &pd, int kind, int *ids_out, floa
 
 pbd_status enqueue_draft(pbd_ctx *c, float *logits) {
     const PassDesc pd = block_pass(c, PK_DRAFT);
-    CK(launch_build_ids(pd, 0, c->s.pending, nullptr, c->D, c->ids, c->st));
-    return run_pass(c, pd, PK_DRAFT, c->draft_ids, logits);
+    const int steps = std::max(1, c->cfg.denoise_steps);
+    for (int s = 0; s < steps; ++s) {
+        // step 1 runs [p, MASK x D]; each further step refills row j (position L+j) with the
+        // previous step's proposal d_j and replaces the proposals with its own
+        CK(launch_build_ids(pd, s == 0 ? 0 : 1, c->s.pending, c->draft_ids, c->D, c->ids, c->st));
+        TRY(run_pass(c, pd, PK_DRAFT, c->draft_ids, s + 1 == steps ? logits : nullptr));
+    }
+    return PBD_OK;
 }
 
 pbd_status enqueue_verify(pbd_ctx *c, const int *drafts, float *logits) {
@@ -547,9 +564,10 @@ double pass_bytes(pbd_ctx *c, int kind, const std::vector<int> &Ls) {
         w += 2.0 * lin_main(k, lin) * lin_K(k, lin);
         lora += 2.0 * k.lora_rank * (lin_K(k, lin) + lin_main(k, lin));
     }
-    double bytes = k.n_layers * (w + (kind == PK_DRAFT ? lora : 0.0));
-    bytes += 2.0 * (2.0 * k.n_layers * k.hidden + 2.0 * k.n_layers * k.head_dim);  // norm gains
-    const double kv_tok = 2.0 * 2.0 * k.n_layers * k.n_kv_heads * k.head_dim;
+    const int nl = draft_pass_layers(c, kind);
+    double bytes = nl * (w + (kind == PK_DRAFT ? lora : 0.0));
+    bytes += 2.0 * (2.0 * nl * k.hidden + 2.0 * nl * k.head_dim);  // norm gains
+    const double kv_tok = 2.0 * 2.0 * nl * k.n_kv_heads * k.head_dim;
     const int rows = kind == PK_DECODE ? 1 : c->D + 1;
     for (int L : Ls) bytes += kv_tok * (L + rows);
     return bytes;
@@ -672,6 +690,7 @@ pbd_status pbd_prefill(pbd_ctx *c, int32_t batch, const int32_t *d_prompt_ids, c
             pd.mask_mode = MASK_CAUSAL;
             pd.ro_first = last ? rows - 1 : 0;
             pd.ro_count = last ? 1 : 0;
+            pd.nl_run = c->cfg.n_layers;
             const std::vector<int> ns(1, (c0 + rows + ATT_SPLIT - 1) / ATT_SPLIT);
             CK(cudaStreamSynchronize(c->st));  // the schedule slot is rewritten per chunk
             TRY(upload_schedule(c, PK_PREFILL, pd, ns));

@@ -32,6 +32,7 @@ struct PassDesc {
     int mask_mode;   // MaskMode
     int ro_first;    // read-out rows per sequence: i in [ro_first, ro_first + ro_count)
     int ro_count;
+    int nl_run;      // decoder layers the pass runs before the final norm (the draft's early exit)
 };
 
 // Paged KV cache: [layer][page][Hkv][PAGE][d] bf16 for K and for V.

@@ -42,6 +42,14 @@ def test_workspace_size_and_config_validation(lib):
     assert lib.pbd_workspace_bytes(C.byref(bad)) == 0
     tiny = pbd.make_config(synth.TINY, 16, 4, 256)
     assert 0 < lib.pbd_workspace_bytes(C.byref(tiny)) < 200_000_000
+    # draft variants: early exit within the depth, at most 8 denoising steps, a 0/1 readout flag
+    var = pbd.make_config(synth.TINY, 16, 4, 256, draft_layers=1, denoise_steps=2, anchored=False)
+    assert lib.pbd_workspace_bytes(C.byref(var)) == lib.pbd_workspace_bytes(C.byref(tiny))
+    for field, value in (("draft_layers", synth.TINY.n_layers + 1), ("draft_layers", -1), ("denoise_steps", 9),
+                         ("draft_unanchored", 2)):
+        bad = pbd.make_config(synth.TINY, 16, 4, 256)
+        setattr(bad, field, value)
+        assert lib.pbd_workspace_bytes(C.byref(bad)) == 0, field
 
 
 def test_create_rejects_bad_arguments_without_gpu(lib):
