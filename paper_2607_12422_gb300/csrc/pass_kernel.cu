@@ -43,6 +43,7 @@ constexpr int CT = 192;            // compute-group threads (warps 2-7)
 constexpr int HALF_ATOMS = 4;      // 64-wide swizzle atoms of one operand staging round (K 256)
 constexpr int MAX_ATOMS = 8;       // atoms per linear item at most (K slice 512)
 constexpr int MAX_SLOT = 12;
+constexpr int CT_PAGES = 32;       // compute thread (warp 3, lane 0) that requests attention pages
 constexpr int RING_SLOTS = 4;      // weight tiles in the ring (64 KiB)
 constexpr int MAX_ROWS = 256;
 
@@ -780,13 +781,30 @@ __device__ __noinline__ void attn_combine(const MKParams &P, int bl, int g, int 
 __device__ __forceinline__ bool att_shared_merge(int nsp) { return nsp <= (int)gridDim.x; }
 __device__ __forceinline__ int att_done(int nsp) { return att_shared_merge(nsp) ? 2 * nsp : nsp + 1; }
 
-// wait for every tile of linear `lin` that holds output features [f0, f1): each of its ks
-// slices counts once when stored and once when its rows are reduced
-__device__ bool wait_tiles(const MKParams &P, int layer, int lin, int f0, int f1) {
-    const int off = P.cl.lin[lin];
-    for (int t = f0 / TILE_ROWS; t <= (f1 - 1) / TILE_ROWS; ++t)
-        if (!spin_until(ctr(P, layer, off + t), 2 * P.ks[lin], P)) return false;
-    return true;
+// 128-row tiles that overlap features [f0, f1)
+__device__ __forceinline__ int tiles_over(int f0, int f1) { return (f1 - 1) / TILE_ROWS - f0 / TILE_ROWS + 1; }
+
+// KV head groups whose q, k or v features overlap q|k|v tile t: [*g0, *g1]
+__device__ __forceinline__ void qkv_tile_groups(const Dims &dm, int t, int *g0, int *g1) {
+    const int grp = dm.Hq / dm.Hkv, qw = dm.Hq * dm.d, kvw = dm.Hkv * dm.d;
+    const int f0 = t * TILE_ROWS, f1 = f0 + TILE_ROWS - 1;  // the tile lies in one of q, k, v
+    if (f0 < qw) {
+        *g0 = f0 / dm.d / grp;
+        *g1 = f1 / dm.d / grp;
+    } else {
+        const int base = f0 < qw + kvw ? qw : qw + kvw;
+        *g0 = (f0 - base) / dm.d;
+        *g1 = (f1 - base) / dm.d;
+    }
+}
+
+// slices stored by the reducers an attention item of group g waits for: every slice of every
+// q, k and v tile that holds a feature of the group
+__device__ __forceinline__ int att_in_target(const MKParams &P, int g) {
+    const Dims &dm = P.dm;
+    const int grp = dm.Hq / dm.Hkv, d = dm.d, qw = dm.Hq * d, kvw = dm.Hkv * d;
+    return P.ks[0] * (tiles_over(g * grp * d, (g + 1) * grp * d) + tiles_over(qw + g * d, qw + (g + 1) * d) +
+                      tiles_over(qw + kvw + g * d, qw + kvw + (g + 1) * d));
 }
 
 // the item's inputs are complete (one thread; false on abort)
@@ -811,22 +829,14 @@ __device__ bool wait_deps(const MKParams &P, const MKItem &it) {
             }
             case 2: return spin_until(ctr(P, l, P.cl.res_o), dm.H / TILE_ROWS * P.ks[1], P);
             default: {
-                // act features [256 s, 256 s + 256) live in gate|up tiles 4s..4s+3
+                // act features [w s, w s + w) live in gate|up tiles (64 features each); each of
+                // their reducers counts once on the slice's counter
                 const int w = P.katoms[3] * KT;
-                const int t0 = (s * w) / 64, t1 = (s * w + w - 1) / 64;
-                for (int t = t0; t <= t1; ++t)
-                    if (!spin_until(ctr(P, l, P.cl.lin[2] + t), 2 * P.ks[2], P)) return false;
-                return true;
+                return spin_until(ctr(P, l, P.cl.act + s), (w / 64) * P.ks[2], P);
             }
         }
     }
-    if (it.op == MK_ATTN) {
-        const int g = it.b, grp = dm.Hq / dm.Hkv, d = dm.d;
-        const int qw = dm.Hq * d, kvw = dm.Hkv * d;
-        return wait_tiles(P, l, 0, g * grp * d, (g + 1) * grp * d) &&
-               wait_tiles(P, l, 0, qw + g * d, qw + (g + 1) * d) &&
-               wait_tiles(P, l, 0, qw + kvw + g * d, qw + kvw + (g + 1) * d);
-    }
+    if (it.op == MK_ATTN) return spin_until(ctr(P, l, P.cl.att_in + it.b), att_in_target(P, it.b), P);
     if (it.op == MK_FINAL) return spin_until(ctr(P, P.pd.nl_run - 1, P.cl.res_dn), dm.H / TILE_ROWS * P.ks[3], P);
     return true;
 }
@@ -953,6 +963,9 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
         const int ct = tid - 64, cw = warp - 2;
         uint32_t li = 0, ai = 0, l8 = 0;
         unsigned long long *tr = P.trace ? P.trace + 8ull * P.cta_off[blockIdx.x] : nullptr;
+        // the attention pages are requested by thread CT_PAGES while thread 0 polls the item's
+        // inputs; att_pend (that thread only): pages requested for a split that has not waited
+        bool att_pend = false;
         for (int i = 0; i < n_my; ++i) {
             const MKItem it = my[i];
             if (tr && ct == 0) {
@@ -961,10 +974,12 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 tr[8 * i] = now;
             }
             const bool att_active = it.op == MK_ATTN && it.c * ATT_SPLIT < P.L[P.pd.b0 + it.a] + P.pd.R;
-            if (att_active && ct == 0) {
-                // pages below the cached length do not depend on this pass: fetch them now
+            if (att_active && ct == CT_PAGES) {
+                // pages below the cached length do not depend on this pass: fetch them now (the
+                // barrier after the input wait orders this before the split's arrival)
                 mbar_expect_tx(&att_bar, attn_pages(P, it.layer, it.a, it.b, it.c, 0, uni, &att_bar, false));
                 attn_pages(P, it.layer, it.a, it.b, it.c, 0, uni, &att_bar, true);
+                att_pend = true;
             }
             if (ct == 0) s_flag = wait_deps(P, it) ? 1 : 0;
             bar_compute();
@@ -1004,6 +1019,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                     unsigned long long *st = tr ? tr + 8 * i : nullptr;
                     attn_split<DH, DRAFT>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st);
                     ++ai;
+                    att_pend = false;
                 }
                 bar_compute();
                 if (tr && ct == 0) tr[8 * i + 2] = globaltimer_ns();
@@ -1128,13 +1144,29 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                     reduce_residual<DRAFT>(P, lin, l, t, cw, lane, s, ks);
                 bar_compute();
                 if (ct == 0) {
-                    red_release_add(c, 1);
+                    // one release per reduction, on the counter its consumers poll
                     if (lin == 1 || lin == 3) red_release_add(ctr(P, l, lin == 1 ? P.cl.res_o : P.cl.res_dn), 1);
+                    if (lin == 0) {
+                        // the attention of every group the tile feeds counts this reduction
+                        int g0, g1;
+                        qkv_tile_groups(P.dm, t, &g0, &g1);
+                        for (int g = g0; g <= g1; ++g) red_release_add(ctr(P, l, P.cl.att_in + g), 1);
+                    }
+                    // the down-projection slice holding the tile's act features counts it
+                    if (lin == 2) red_release_add(ctr(P, l, P.cl.act + t * 64 / (P.katoms[3] * KT)), 1);
                 }
                 if (tr && ct == 0) tr[8 * i + 7] = globaltimer_ns();
             }
         }
         if (tr && ct == 0 && n_my > 0) tr[8 * (n_my - 1) + 3] = globaltimer_ns();
+        if (ct == CT_PAGES && att_pend) {
+            // the pass ended before the split waited for its pages: complete the phase's arrival
+            // and let the copies land (bounded) before the shared memory is released
+            mbarrier_arrive_one(&att_bar);
+            const uint64_t t0 = globaltimer_ns();
+            while (!mbar_try_wait(smem_u32(&att_bar), ai & 1) && globaltimer_ns() - t0 < WAIT_LIMIT_NS) {
+            }
+        }
     }
     tc_fence_before();
     __syncthreads();
@@ -1172,7 +1204,9 @@ void mk_counter_layout(const Dims &dm, int max_nb, CounterLayout *cl) {
     cl->res_o = nq + no + ng + nd;
     cl->res_dn = cl->res_o + 1;
     cl->att = cl->res_dn + 1;
-    cl->per_layer = cl->att + max_nb * dm.Hkv;
+    cl->att_in = cl->att + max_nb * dm.Hkv;
+    cl->act = cl->att_in + dm.Hkv;
+    cl->per_layer = cl->act + dm.I / (mk_slice_atoms(3, dm.I) * KT);
     cl->total = cl->global + dm.nl * cl->per_layer;
 }
 

@@ -79,9 +79,11 @@ struct CounterLayout {
     int embed;      // rows embedded
     int global;     // first per-layer counter
     int per_layer;  // counters per layer
-    int lin[4];     // per-tile slice arrivals (+1 once reduced), per linear
+    int lin[4];     // per-tile stored slices (the split reduction waits for all of them), per linear
     int res_o, res_dn;  // residual tiles finished after o / down
     int att;        // per (sequence, KV head): split items done (+1 once merged)
+    int att_in;     // per KV head: reduced q|k|v tile slices that its attention reads
+    int act;        // per down-projection K slice: reduced gate|up tile slices it reads
     int total;
 };
 
