@@ -18,16 +18,21 @@
 //               while building the activation tile in the swizzle layout), the TMEM epilogue
 //               (warps 4-7, one per TMEM lane quarter), attention, split reductions.
 //
-// A linear is split along K into 256-wide slices (fixed per linear, independent of the row
-// count).  Each slice item stores fp32 partial sums; the CTA that completes a tile last (atomic
-// counter) adds the slices in slice order and finishes the step for that tile:
+// A linear is split along K into 256-wide slices (512 for gate|up; fixed per linear, independent
+// of the row count).  Each slice item stores its fp32 partial sums as 64-bit words tagged with
+// the (pass, layer); the tile's slice items sit on distinct CTAs, and each of them then reduces
+// every ks-th row of the tile, adding the slices in slice order as their tagged words arrive
+// (no completion counter between the slices), and finishes the step for those rows:
 //   q|k|v tile   -> + adapter delta, bf16, per-head RMSNorm, RoPE, q buffer / paged K, V
 //   o tile       -> + adapter delta, residual add into h, per-tile sum of squares of h
 //   gate|up tile -> + adapter delta, SiLU(gate) * up into the act buffer (gate/up interleaved)
 //   down tile    -> + adapter delta, residual add into h, per-tile sum of squares of h
-//   adapter tile -> u = bf16(x A^T) for the tiles above (scheduled first in every phase)
-// Attention items cover (sequence, KV head, 128-key split); the last split of a head group
-// merges the splits into the attention output.  RMSNorm statistics are summed per 128-feature
+// The adapter's A rows form one extra tile whose partials u = x A^T the reducers above sum
+// themselves.  Each reduction then counts once, with release semantics, on the counter its
+// consumers poll (attention inputs per KV head, a down-projection K slice, the residual).
+// Attention items cover (sequence, KV head, 128-key split); when the splits sit on distinct
+// CTAs they wait for one another and each merges a share of the rows, else the last one
+// merges all.  RMSNorm statistics are summed per 128-feature
 // tile in one fixed order, so every row's arithmetic is independent of the pass it is in.
 #include <algorithm>
 #include <cmath>
@@ -43,6 +48,7 @@ constexpr int CT = 192;            // compute-group threads (warps 2-7)
 constexpr int HALF_ATOMS = 4;      // 64-wide swizzle atoms of one operand staging round (K 256)
 constexpr int MAX_ATOMS = 8;       // atoms per linear item at most (K slice 512)
 constexpr int MAX_SLOT = 12;
+constexpr int MK_STARTED = 1;      // global counter slot: CTAs that have read the pass counter
 constexpr int CT_PAGES = 32;       // compute thread (warp 3, lane 0) that requests attention pages
 constexpr int RING_SLOTS = 4;      // weight tiles in the ring (64 KiB)
 constexpr int MAX_ROWS = 256;
@@ -61,6 +67,16 @@ __device__ __forceinline__ int ld_relaxed(const int *p) {
     int v;
     asm volatile("ld.relaxed.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
+}
+
+// single-copy-atomic 64-bit accesses of the tagged partials
+__device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long long *p) {
+    unsigned long long v;
+    asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(v) : "l"(p));
+    return v;
+}
+__device__ __forceinline__ void st_relaxed_u64(unsigned long long *p, unsigned long long v) {
+    asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(v));
 }
 
 __device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
@@ -89,7 +105,8 @@ struct MKParams {
     const int *L;
     const int *ids;
     // scratch
-    float *part[4];
+    unsigned long long *part[4];  // split-K partials: fp32 bits | (pass, layer) tag << 32 (see sum_parts)
+    int *epoch;                   // tag counter: layer l of a pass tags its partials *epoch + 1 + l
     int part_rows;
     bf16 *h, *q, *attn, *act, *x_ro;
     float *ss;                 // [rows][H/128]
@@ -118,23 +135,6 @@ __device__ bool spin_until(const int *c, int target, const MKParams &P) {
     for (;;) {
         for (int i = 0; i < 8; ++i) {
             if (ld_acquire(c) >= target) return true;
-            __nanosleep(40);
-        }
-        if (aborted(P)) return false;
-        if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
-            raise_abort(P, DEV_TIMEOUT_DEP);
-            return false;
-        }
-    }
-}
-
-// one thread: wait until *c1 >= t1 and *c2 >= t2, both polled in each round (bounded)
-__device__ bool spin_until2(const int *c1, int t1, const int *c2, int t2, const MKParams &P) {
-    const uint64_t t0 = globaltimer_ns();
-    for (;;) {
-        for (int i = 0; i < 8; ++i) {
-            const int v1 = ld_acquire(c1), v2 = ld_acquire(c2);
-            if (v1 >= t1 && v2 >= t2) return true;
             __nanosleep(40);
         }
         if (aborted(P)) return false;
@@ -239,24 +239,54 @@ __device__ __forceinline__ void share_u(float lane_sum, int base, float (&u)[MAX
 
 // Sums of the K-slice partials of E features of row m, slices added in order; loads go out
 // in batches of S slices (every load of a batch in flight before the first add).
+// Each partial is one 64-bit word, the fp32 value and the tag of the (pass, layer) that stored
+// it, written and read with single-copy-atomic accesses: a word carrying this layer's tag holds
+// this layer's value, so the sum polls the words themselves instead of a completion counter.
+// Words still carrying an older tag are read again (bounded; on timeout or abort the pass is lost).
 template <int E, int S>
-__device__ __forceinline__ void sum_parts(const MKParams &P, int lin, int m, const int *f, float *out) {
+__device__ __forceinline__ void sum_parts(const MKParams &P, int lin, int m, const int *f, float *out, uint32_t tag) {
     const int nt = P.n_main[lin] + P.lora_rows[lin];
-    const float *p = P.part[lin] + (size_t)m * nt;
+    const unsigned long long *p = P.part[lin] + (size_t)m * nt;
     const size_t stride = (size_t)P.part_rows * nt;
     const int ks = P.ks[lin];
     for (int s0 = 0; s0 < ks; s0 += S) {
-        float v[E][S];
+        unsigned long long v[E][S];
 #pragma unroll
         for (int s = 0; s < S; ++s)
 #pragma unroll
-            for (int e = 0; e < E; ++e) v[e][s] = s0 + s < ks ? __ldcg(p + (s0 + s) * stride + f[e]) : 0.f;
+            for (int e = 0; e < E; ++e)
+                v[e][s] = s0 + s < ks ? ld_relaxed_u64(p + (s0 + s) * stride + f[e]) : (unsigned long long)tag << 32;
+        bool stale = false;
+#pragma unroll
+        for (int s = 0; s < S; ++s)
+#pragma unroll
+            for (int e = 0; e < E; ++e) stale |= (uint32_t)(v[e][s] >> 32) != tag;
+        if (stale) {
+            const uint64_t t0 = globaltimer_ns();
+            while (stale) {
+                __nanosleep(32);
+                stale = false;
+#pragma unroll
+                for (int s = 0; s < S; ++s)
+#pragma unroll
+                    for (int e = 0; e < E; ++e)
+                        if ((uint32_t)(v[e][s] >> 32) != tag) {
+                            v[e][s] = ld_relaxed_u64(p + (s0 + s) * stride + f[e]);
+                            stale |= (uint32_t)(v[e][s] >> 32) != tag;
+                        }
+                if (stale && (aborted(P) || globaltimer_ns() - t0 > WAIT_LIMIT_NS)) {
+                    if (!aborted(P)) raise_abort(P, DEV_TIMEOUT_DEP);
+                    break;
+                }
+            }
+        }
 #pragma unroll
         for (int e = 0; e < E; ++e) {
 #pragma unroll
             for (int s = 0; s < S; ++s) {
                 if (s0 + s >= ks) break;
-                out[e] = (s0 + s == 0) ? v[e][s] : __fadd_rn(out[e], v[e][s]);
+                const float x = __uint_as_float((uint32_t)v[e][s]);
+                out[e] = (s0 + s == 0) ? x : __fadd_rn(out[e], x);
             }
         }
     }
@@ -348,7 +378,8 @@ __device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int 
 
 // q|k|v tile: adapter delta, bf16, per-head RMSNorm + RoPE for q and k, store q / paged K, V
 template <int DH, bool AD>
-__device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, int cw, int lane, int m0, int mstep) {
+__device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, int cw, int lane, int m0, int mstep,
+                                       uint32_t tag) {
     constexpr int E = DH / 32;
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r;
@@ -373,7 +404,7 @@ __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, 
 #pragma unroll
             for (int j = 0; j < E; ++j) br[j] = load_brow(lb + (size_t)f[j] * r, r);
         float y[E + 1];
-        sum_parts<E + (AD ? 1 : 0), 8>(P, 0, m, f, y);
+        sum_parts<E + (AD ? 1 : 0), AD ? 4 : 8>(P, 0, m, f, y, tag);
         float u[MAX_RANK];
         if (AD) share_u(y[E], 0, u);
 #pragma unroll
@@ -427,7 +458,7 @@ __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, 
 // o or down tile: adapter delta, residual add into h, per-tile sum of squares
 template <bool AD>
 __device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int layer, int tile, int cw, int lane, int m0,
-                                             int mstep) {
+                                             int mstep, uint32_t tag) {
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r, H = dm.H, nt = H / TILE_ROWS;
     const bf16 *lb = P.lora_b[lin] + (size_t)layer * P.lb_stride[lin];
@@ -447,7 +478,7 @@ __device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int lay
             hv[e] = bf2f(ldcg_bf(P.h + (size_t)m * H + f[e]));
         }
         f[4] = P.n_main[lin] + (lane < r ? lane : 0);
-        sum_parts<AD ? 5 : 4, 8>(P, lin, m, f, acc);
+        sum_parts<AD ? 5 : 4, AD ? 4 : 8>(P, lin, m, f, acc, tag);
         float u[MAX_RANK];
         if (AD) share_u(acc[4], 0, u);
         float v[4];
@@ -464,7 +495,8 @@ __device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int lay
 
 // gate|up tile (rows 0-63 gate features 64t.., rows 64-127 up features 64t..): SiLU(gate)*up
 template <bool AD>
-__device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, int cw, int lane, int m0, int mstep) {
+__device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, int cw, int lane, int m0, int mstep,
+                                      uint32_t tag) {
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r, I = dm.I;
     const bf16 *lb = P.lora_b[2] + (size_t)layer * P.lb_stride[2];
@@ -483,7 +515,7 @@ __device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, i
         const int f[5] = {tile * TILE_ROWS + lane, tile * TILE_ROWS + lane + 32, tile * TILE_ROWS + 64 + lane,
                           tile * TILE_ROWS + 96 + lane, P.n_main[2] + (lane < 2 * r ? lane : 0)};
         float ug[MAX_RANK], uu[MAX_RANK], s[5];
-        sum_parts<AD ? 5 : 4, 2>(P, 2, m, f, s);
+        sum_parts<AD ? 5 : 4, 2>(P, 2, m, f, s, tag);
         if (AD) {
             share_u(s[4], 0, ug);
             share_u(s[4], r, uu);
@@ -856,6 +888,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
     // compute-group flags: each is written by thread 0 and read by all after a barrier, and is
     // not written again before every thread has passed at least one more barrier
     __shared__ int s_flag, s_red, s_ok;
+    __shared__ uint32_t s_tag;  // this pass's partial-sum tag
     __shared__ float s_rms[MAX_ROWS];
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -863,6 +896,11 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
     const int n_my = P.cta_off[blockIdx.x + 1] - P.cta_off[blockIdx.x];
 
     if (tid == 0) {
+        // the previous pass on this stream has finished: its counter advance is visible. Layer l
+        // of this pass tags its partials s_tag + l; the buffers are reused by every layer and
+        // pass, so a tag identifies both (acquire: read before the arrival below)
+        s_tag = (uint32_t)ld_acquire(P.epoch) + 1u;
+        atomicAdd(P.cnt + MK_STARTED, 1);
         for (int i = 0; i < P.nslot; ++i) {
             mbar_init(&full[i], 1);
             mbar_init(&empty[i], 1);
@@ -1101,10 +1139,12 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                             tmem_ld_32cols(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)c0, v);
                             tmem_ld_wait();
                             if (row < rows_valid) {
-                                float *dst = P.part[lin] + ((size_t)s * P.part_rows + c0) * n_total + t * TILE_ROWS + row;
+                                unsigned long long *dst =
+                                    P.part[lin] + ((size_t)s * P.part_rows + c0) * n_total + t * TILE_ROWS + row;
+                                const unsigned long long tg = (unsigned long long)(s_tag + l) << 32;
 #pragma unroll
                                 for (int j = 0; j < 32; ++j)
-                                    if (c0 + j < P.pd.M) dst[(size_t)j * n_total] = __uint_as_float(v[j]);
+                                    if (c0 + j < P.pd.M) st_relaxed_u64(dst + (size_t)j * n_total, tg | v[j]);
                             }
                         }
                     }
@@ -1114,34 +1154,23 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 bar_compute();
                 if (tr && ct == 0) tr[8 * i + 2] = globaltimer_ns();
                 // The tile's slices are consecutive items of the round-robin schedule, so they sit on
-                // distinct CTAs that all reach them: each CTA announces its stored slice, waits for the
-                // others, then reduces rows s, s + ks, ... of the tile (s = its slice).
-                int *c = ctr(P, l, P.cl.lin[lin] + t);
+                // distinct CTAs that all reach them: each CTA stores its tagged slice partials, then
+                // reduces rows s, s + ks, ... of the tile (s = its slice), reading the other slices'
+                // partials as they arrive. The adapter tile's partials are summed by the main tiles'
+                // reducers themselves.
                 const int ks = P.ks[lin];
+                if (tr && ct == 0) tr[8 * i + 6] = globaltimer_ns();
                 if (lt) {
-                    // the adapter tile's partials are summed by the main tiles' reducers themselves
-                    if (ct == 0) red_release_add(c, 1);
-                    if (tr && ct == 0) tr[8 * i + 6] = tr[8 * i + 7] = globaltimer_ns();
+                    if (tr && ct == 0) tr[8 * i + 7] = globaltimer_ns();
                     continue;
                 }
-                if (ct == 0) {
-                    red_release_add(c, 1);
-                    if (tr) tr[8 * i + 6] = globaltimer_ns();
-                    // with the adapter, every slice of the adapter tile must be stored too (both
-                    // counters polled together)
-                    const bool ok = (DRAFT && P.lora_rows[lin] > 0)
-                                        ? spin_until2(c, ks, ctr(P, l, P.cl.lin[lin] + P.n_main[lin] / TILE_ROWS), ks, P)
-                                        : spin_until(c, ks, P);
-                    s_ok = ok ? 1 : 0;
-                }
-                bar_compute();
-                if (!s_ok) break;
+                const uint32_t tag = s_tag + l;
                 if (lin == 0) {
-                    reduce_qkv<DH, DRAFT>(P, l, t, cw, lane, s, ks);
+                    reduce_qkv<DH, DRAFT>(P, l, t, cw, lane, s, ks, tag);
                 } else if (lin == 2)
-                    reduce_gu<DRAFT>(P, l, t, cw, lane, s, ks);
+                    reduce_gu<DRAFT>(P, l, t, cw, lane, s, ks, tag);
                 else
-                    reduce_residual<DRAFT>(P, lin, l, t, cw, lane, s, ks);
+                    reduce_residual<DRAFT>(P, lin, l, t, cw, lane, s, ks, tag);
                 bar_compute();
                 if (ct == 0) {
                     // one release per reduction, on the counter its consumers poll
@@ -1171,6 +1200,13 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
     tc_fence_before();
     __syncthreads();
     if (warp == 0) tmem_dealloc(tmem, P.tmem_cols);
+    if (blockIdx.x == 0 && tid == 0) {
+        // once every CTA has read the pass counter (bounded), advance it for the next pass
+        const uint64_t t0 = globaltimer_ns();
+        while (ld_relaxed(P.cnt + MK_STARTED) < (int)gridDim.x && globaltimer_ns() - t0 < WAIT_LIMIT_NS) {
+        }
+        asm volatile("st.relaxed.gpu.global.b32 [%0], %1;" ::"l"(P.epoch), "r"((int)(s_tag + P.dm.nl - 1)) : "memory");
+    }
 }
 
 // ------------------------------------------------------------------ host side
@@ -1191,17 +1227,9 @@ int mk_grid_size() {
 }
 
 void mk_counter_layout(const Dims &dm, int max_nb, CounterLayout *cl) {
-    const int nq = (dm.Hq + 2 * dm.Hkv) * dm.d / TILE_ROWS + 1;
-    const int no = dm.H / TILE_ROWS + 1;
-    const int ng = 2 * dm.I / TILE_ROWS + 1;
-    const int nd = dm.H / TILE_ROWS + 1;
     cl->embed = 0;
     cl->global = 4;
-    cl->lin[0] = 0;
-    cl->lin[1] = nq;
-    cl->lin[2] = nq + no;
-    cl->lin[3] = nq + no + ng;
-    cl->res_o = nq + no + ng + nd;
+    cl->res_o = 0;
     cl->res_dn = cl->res_o + 1;
     cl->att = cl->res_dn + 1;
     cl->att_in = cl->att + max_nb * dm.Hkv;
@@ -1293,6 +1321,7 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
         P.lora_b[i] = static_cast<const bf16 *>(L.lora_b[i]);
         P.lb_stride[i] = L.lb_stride[i];
         P.part[i] = L.part[i];
+        P.epoch = L.epoch;
     }
     P.attn_norm = static_cast<const bf16 *>(L.attn_norm);
     P.mlp_norm = static_cast<const bf16 *>(L.mlp_norm);

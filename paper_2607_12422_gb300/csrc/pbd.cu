@@ -87,7 +87,9 @@ struct pbd_ctx {
     int *page_table;
     // scratch
     void *h, *q, *attn, *act, *x_ro;
-    float *part[4], *ss, *o_part;
+    unsigned long long *part[4];  // tagged split-K partials of the pass kernel
+    size_t part_bytes[4];
+    float *ss, *o_part;
     float2 *ml_part;
     float *tile_max;
     int *tile_arg;
@@ -217,7 +219,8 @@ size_t layout(pbd_ctx *c, void *base) {
     c->status = (int *)bp.take(64);
     c->s.all_done = c->status + 1;
     c->s.round = c->status + 2;
-    c->cnt = (int *)bp.take(sizeof(int) * (size_t)(c->cl.total + 1));
+    // abort flag, the pass counters, then the pass counter that tags split-K partials
+    c->cnt = (int *)bp.take(sizeof(int) * (size_t)(c->cl.total + 2));
     c->s.stats = (long long *)bp.take(3 * sizeof(long long));
     c->s.L = (int *)bp.take(sizeof(int) * B);
     c->s.pending = (int *)bp.take(sizeof(int) * B);
@@ -276,8 +279,9 @@ size_t layout(pbd_ctx *c, void *base) {
     c->x_ro = bp.take(e2 * c->ro_alloc * H);
     c->ss = (float *)bp.take(sizeof(float) * RA * (H / TILE_ROWS));
     for (int lin = 0; lin < 4; ++lin) {
-        c->part[lin] = (float *)bp.take(sizeof(float) * (size_t)(lin_K(k, lin) / 256) * RA *
-                                        (lin_main(k, lin) + lin_lora(k, lin)));
+        c->part_bytes[lin] = sizeof(unsigned long long) * (size_t)(lin_K(k, lin) / 256) * RA *
+                             (lin_main(k, lin) + lin_lora(k, lin));
+        c->part[lin] = (unsigned long long *)bp.take(c->part_bytes[lin]);
     }
     c->o_part = (float *)bp.take(sizeof(float) * (size_t)RA * Hq * c->n_splits * ATT_SUBS * d);
     c->ml_part = (float2 *)bp.take(sizeof(float2) * (size_t)RA * Hq * c->n_splits * ATT_SUBS);
@@ -448,6 +452,7 @@ MKLaunch make_launch(pbd_ctx *c, const PassDesc &pd, int kind) {
         L.lb_stride[lin] = (size_t)w0.n_main * k.lora_rank;
         L.part[lin] = c->part[lin];
     }
+    L.epoch = c->cnt + c->cl.total + 1;
     L.attn_norm = c->attn_norm;
     L.mlp_norm = c->mlp_norm;
     L.q_norm = c->q_norm;
@@ -629,7 +634,10 @@ pbd_status pbd_create(const pbd_config *cfg, const pbd_base_weights *base, const
         return s;
     }
     const size_t kv_bytes = (size_t)cfg->n_layers * c->n_pages * cfg->n_kv_heads * PAGE * cfg->head_dim * 2;
-    if ((e = cudaMemsetAsync(c->kv.k, 0, kv_bytes, c->st)) != cudaSuccess ||
+    // the split-K partials start with tag 0, below every pass's tag (the pass counter starts at 0)
+    for (int lin = 0; lin < 4 && e == cudaSuccess; ++lin) e = cudaMemsetAsync(c->part[lin], 0, c->part_bytes[lin], c->st);
+    if (e != cudaSuccess || (e = cudaMemsetAsync(c->cnt, 0, sizeof(int) * (size_t)(c->cl.total + 2), c->st)) != cudaSuccess ||
+        (e = cudaMemsetAsync(c->kv.k, 0, kv_bytes, c->st)) != cudaSuccess ||
         (e = cudaMemsetAsync(c->kv.v, 0, kv_bytes, c->st)) != cudaSuccess ||
         (e = cudaMemsetAsync(c->status, 0, 64, c->st)) != cudaSuccess ||
         (e = cudaStreamSynchronize(c->st)) != cudaSuccess) {

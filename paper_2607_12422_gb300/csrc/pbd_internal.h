@@ -77,9 +77,8 @@ struct __align__(16) MKItem {
 // Offsets of the pass's completion counters (ints, zeroed before every pass).
 struct CounterLayout {
     int embed;      // rows embedded
-    int global;     // first per-layer counter
+    int global;     // first per-layer counter (slots before it: embed, CTAs started)
     int per_layer;  // counters per layer
-    int lin[4];     // per-tile stored slices (the split reduction waits for all of them), per linear
     int res_o, res_dn;  // residual tiles finished after o / down
     int att;        // per (sequence, KV head): split items done (+1 once merged)
     int att_in;     // per KV head: reduced q|k|v tile slices that its attention reads
@@ -108,7 +107,8 @@ struct MKLaunch {
     KVCache kv;
     const int *Lbuf;
     const int *ids;
-    float *part[4];
+    unsigned long long *part[4];  // split-K partials, tagged with the pass counter
+    int *epoch;                   // pass counter (device)
     int part_rows;
     void *h, *q, *attn, *act, *x_ro;
     float *ss;
