@@ -78,6 +78,12 @@ __device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long
 __device__ __forceinline__ void st_relaxed_u64(unsigned long long *p, unsigned long long v) {
     asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(v));
 }
+__device__ __forceinline__ bool tag_is(unsigned long long w, uint32_t tag) { return (uint32_t)(w >> 32) == tag; }
+// 16-byte load, single-copy atomic per 64-bit element
+__device__ __forceinline__ void ld_relaxed_2u64(const unsigned long long *p, unsigned long long &a,
+                                                unsigned long long &b) {
+    asm volatile("ld.relaxed.gpu.global.v2.b64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "l"(p));
+}
 
 __device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
@@ -108,7 +114,8 @@ struct MKParams {
     unsigned long long *part[4];  // split-K partials: fp32 bits | (pass, layer) tag << 32 (see sum_parts)
     int *epoch;                   // tag counter: layer l of a pass tags its partials *epoch + 1 + l
     int part_rows;
-    bf16 *h, *q, *attn, *act, *x_ro;
+    bf16 *h, *q, *attn, *x_ro;
+    unsigned long long *act;   // SiLU(gate) * up: words of two bf16 (features 2j, 2j+1) | tag << 32
     float *ss;                 // [rows][H/128]
     float *o_part;
     float2 *ml_part;
@@ -333,7 +340,7 @@ __device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int 
     const int cpr = na * (KT / 8);  // 16-byte chunks per row
     const bool norm = (lin == 0 || lin == 2);
     const bf16 *gain = lin == 0 ? P.attn_norm + (size_t)layer * P.dm.H : P.mlp_norm + (size_t)layer * P.dm.H;
-    const bf16 *src = norm ? P.h : (lin == 1 ? P.attn : P.act);
+    const bf16 *src = norm ? P.h : P.attn;  // the down projection's operand: build_b_act
     const int ld = norm ? P.dm.H : (lin == 1 ? P.dm.Hq * P.dm.d : P.dm.I);
     const int chunks = M * cpr;
     uint4 xv[U], gv[U];
@@ -372,6 +379,49 @@ __device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int 
                 for (int e = 0; e < 8; ++e) oe[e] = f2bf(__fmul_rn(bf2f(ge[e]), rbf(__fmul_rn(bf2f(he[e]), rs))));
             }
             *reinterpret_cast<uint4 *>(sb + (size_t)atom * P.bn * 128 + m * 128 + ((cc ^ (m & 7)) << 4)) = val;
+        }
+    }
+}
+
+// The down projection's activation tile from the tagged act words of this layer's gate|up
+// reductions (same layout as build_b): every 16-byte chunk of 8 features is four words, read
+// again until all carry the tag (bounded).  No completion counter precedes it.
+__device__ __noinline__ void build_b_act(const MKParams &P, int slice, uint8_t *sb, int ct, uint32_t tag) {
+    constexpr int U = 4;  // chunks in flight per thread
+    const int M = P.pd.M, ld = P.dm.I;
+    const int k0 = slice * P.katoms[3] * KT;
+    const int cpr = P.katoms[3] * (KT / 8);  // 16-byte chunks per row
+    const int chunks = M * cpr;
+    for (int q0 = ct; q0 < chunks; q0 += U * CT) {
+        unsigned long long tw[U][4];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int q = q0 + u * CT;
+            if (q < chunks) {
+                const unsigned long long *w = P.act + ((size_t)(q / cpr) * ld + k0 + (q % cpr) * 8) / 2;
+                ld_relaxed_2u64(w, tw[u][0], tw[u][1]);
+                ld_relaxed_2u64(w + 2, tw[u][2], tw[u][3]);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int q = q0 + u * CT;
+            if (q >= chunks) break;
+            const int m = q / cpr, c = q % cpr;
+            const unsigned long long *w = P.act + ((size_t)m * ld + k0 + c * 8) / 2;
+            const uint64_t t0 = globaltimer_ns();
+            while (!(tag_is(tw[u][0], tag) && tag_is(tw[u][1], tag) && tag_is(tw[u][2], tag) && tag_is(tw[u][3], tag))) {
+                if (aborted(P) || globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
+                    if (!aborted(P)) raise_abort(P, DEV_TIMEOUT_DEP);
+                    break;
+                }
+                __nanosleep(32);
+                ld_relaxed_2u64(w, tw[u][0], tw[u][1]);
+                ld_relaxed_2u64(w + 2, tw[u][2], tw[u][3]);
+            }
+            const int atom = c >> 3, cc = c & 7;
+            *reinterpret_cast<uint4 *>(sb + (size_t)atom * P.bn * 128 + m * 128 + ((cc ^ (m & 7)) << 4)) =
+                make_uint4((uint32_t)tw[u][0], (uint32_t)tw[u][1], (uint32_t)tw[u][2], (uint32_t)tw[u][3]);
         }
     }
 }
@@ -531,7 +581,11 @@ __device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, i
             g = rbf(g);
             up = rbf(up);
             const float sg = __fdiv_rn(g, __fadd_rn(1.0f, expf(-g)));
-            P.act[(size_t)m * I + a] = f2bf(__fmul_rn(sg, up));
+            // features a (even lane) and a + 1 (odd neighbour) go out as one tagged word
+            const uint32_t bits = __bfloat16_as_ushort(f2bf(__fmul_rn(sg, up)));
+            const uint32_t hi = __shfl_down_sync(0xffffffffu, bits, 1);
+            if ((lane & 1) == 0)
+                st_relaxed_u64(P.act + ((size_t)m * I + a) / 2, ((unsigned long long)tag << 32) | (hi << 16) | bits);
         }
     }
 }
@@ -860,12 +914,10 @@ __device__ bool wait_deps(const MKParams &P, const MKItem &it) {
                 return true;
             }
             case 2: return spin_until(ctr(P, l, P.cl.res_o), dm.H / TILE_ROWS * P.ks[1], P);
-            default: {
-                // act features [w s, w s + w) live in gate|up tiles (64 features each); each of
-                // their reducers counts once on the slice's counter
-                const int w = P.katoms[3] * KT;
-                return spin_until(ctr(P, l, P.cl.act + s), (w / 64) * P.ks[2], P);
-            }
+            default:
+                // act words carry the tag of the gate|up reduction that wrote them: the operand
+                // staging polls them itself
+                return true;
         }
     }
     if (it.op == MK_ATTN) return spin_until(ctr(P, l, P.cl.att_in + it.b), att_in_target(P, it.b), P);
@@ -1091,7 +1143,10 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 const int lin = it.lin, l = it.layer, t = it.a, s = it.b;
                 const int na = P.katoms[lin];
                 if (na <= HALF_ATOMS) {
-                    build_b(P, lin, l, s, uni, s_rms, ct, 0, na, true);
+                    if (lin == 3)
+                        build_b_act(P, s, uni, ct, s_tag + l);
+                    else
+                        build_b(P, lin, l, s, uni, s_rms, ct, 0, na, true);
                     fence_proxy_async();
                     bar_compute();
                     if (ct == 0) mbarrier_arrive_one(&b_full[0]);
@@ -1181,8 +1236,6 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                         qkv_tile_groups(P.dm, t, &g0, &g1);
                         for (int g = g0; g <= g1; ++g) red_release_add(ctr(P, l, P.cl.att_in + g), 1);
                     }
-                    // the down-projection slice holding the tile's act features counts it
-                    if (lin == 2) red_release_add(ctr(P, l, P.cl.act + t * 64 / (P.katoms[3] * KT)), 1);
                 }
                 if (tr && ct == 0) tr[8 * i + 7] = globaltimer_ns();
             }
@@ -1233,8 +1286,7 @@ void mk_counter_layout(const Dims &dm, int max_nb, CounterLayout *cl) {
     cl->res_dn = cl->res_o + 1;
     cl->att = cl->res_dn + 1;
     cl->att_in = cl->att + max_nb * dm.Hkv;
-    cl->act = cl->att_in + dm.Hkv;
-    cl->per_layer = cl->act + dm.I / (mk_slice_atoms(3, dm.I) * KT);
+    cl->per_layer = cl->att_in + dm.Hkv;
     cl->total = cl->global + dm.nl * cl->per_layer;
 }
 
@@ -1339,7 +1391,7 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
     P.h = static_cast<bf16 *>(L.h);
     P.q = static_cast<bf16 *>(L.q);
     P.attn = static_cast<bf16 *>(L.attn);
-    P.act = static_cast<bf16 *>(L.act);
+    P.act = static_cast<unsigned long long *>(L.act);
     P.x_ro = static_cast<bf16 *>(L.x_ro);
     P.ss = L.ss;
     P.o_part = L.o_part;

@@ -89,6 +89,7 @@ struct pbd_ctx {
     void *h, *q, *attn, *act, *x_ro;
     unsigned long long *part[4];  // tagged split-K partials of the pass kernel
     size_t part_bytes[4];
+    size_t act_bytes;
     float *ss, *o_part;
     float2 *ml_part;
     float *tile_max;
@@ -275,7 +276,8 @@ size_t layout(pbd_ctx *c, void *base) {
     c->h = bp.take(e2 * RA * H);
     c->q = bp.take(e2 * RA * Hq * d);
     c->attn = bp.take(e2 * RA * Hq * d);
-    c->act = bp.take(e2 * RA * I);
+    c->act_bytes = sizeof(unsigned long long) * RA * (I / 2);  // tagged words of two bf16
+    c->act = bp.take(c->act_bytes);
     c->x_ro = bp.take(e2 * c->ro_alloc * H);
     c->ss = (float *)bp.take(sizeof(float) * RA * (H / TILE_ROWS));
     for (int lin = 0; lin < 4; ++lin) {
@@ -636,6 +638,7 @@ pbd_status pbd_create(const pbd_config *cfg, const pbd_base_weights *base, const
     const size_t kv_bytes = (size_t)cfg->n_layers * c->n_pages * cfg->n_kv_heads * PAGE * cfg->head_dim * 2;
     // the split-K partials start with tag 0, below every pass's tag (the pass counter starts at 0)
     for (int lin = 0; lin < 4 && e == cudaSuccess; ++lin) e = cudaMemsetAsync(c->part[lin], 0, c->part_bytes[lin], c->st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(c->act, 0, c->act_bytes, c->st);
     if (e != cudaSuccess || (e = cudaMemsetAsync(c->cnt, 0, sizeof(int) * (size_t)(c->cl.total + 2), c->st)) != cudaSuccess ||
         (e = cudaMemsetAsync(c->kv.k, 0, kv_bytes, c->st)) != cudaSuccess ||
         (e = cudaMemsetAsync(c->kv.v, 0, kv_bytes, c->st)) != cudaSuccess ||

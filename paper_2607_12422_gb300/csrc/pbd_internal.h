@@ -82,7 +82,6 @@ struct CounterLayout {
     int res_o, res_dn;  // residual tiles finished after o / down
     int att;        // per (sequence, KV head): split items done (+1 once merged)
     int att_in;     // per KV head: reduced q|k|v tile slices that its attention reads
-    int act;        // per down-projection K slice: reduced gate|up tile slices it reads
     int total;
 };
 
