@@ -270,7 +270,7 @@ __device__ __forceinline__ void sum_parts(const MKParams &P, int lin, int m, con
             for (int e = 0; e < E; ++e) stale |= (uint32_t)(v[e][s] >> 32) != tag;
         if (stale) {
             const uint64_t t0 = globaltimer_ns();
-            while (stale) {
+            for (int round = 1; stale; ++round) {
                 __nanosleep(32);
                 stale = false;
 #pragma unroll
@@ -281,7 +281,8 @@ __device__ __forceinline__ void sum_parts(const MKParams &P, int lin, int m, con
                             v[e][s] = ld_relaxed_u64(p + (s0 + s) * stride + f[e]);
                             stale |= (uint32_t)(v[e][s] >> 32) != tag;
                         }
-                if (stale && (aborted(P) || globaltimer_ns() - t0 > WAIT_LIMIT_NS)) {
+                // the abort flag and the time limit every 8 rounds (each check is an L2 round trip)
+                if (stale && (round & 7) == 0 && (aborted(P) || globaltimer_ns() - t0 > WAIT_LIMIT_NS)) {
                     if (!aborted(P)) raise_abort(P, DEV_TIMEOUT_DEP);
                     break;
                 }
@@ -394,6 +395,7 @@ __device__ __noinline__ void build_b_act(const MKParams &P, int slice, uint8_t *
     const int chunks = M * cpr;
     for (int q0 = ct; q0 < chunks; q0 += U * CT) {
         unsigned long long tw[U][4];
+        const unsigned long long none = (unsigned long long)tag << 32;
 #pragma unroll
         for (int u = 0; u < U; ++u) {
             const int q = q0 + u * CT;
@@ -401,6 +403,35 @@ __device__ __noinline__ void build_b_act(const MKParams &P, int slice, uint8_t *
                 const unsigned long long *w = P.act + ((size_t)(q / cpr) * ld + k0 + (q % cpr) * 8) / 2;
                 ld_relaxed_2u64(w, tw[u][0], tw[u][1]);
                 ld_relaxed_2u64(w + 2, tw[u][2], tw[u][3]);
+            } else {
+                tw[u][0] = tw[u][1] = tw[u][2] = tw[u][3] = none;
+            }
+        }
+        // stale words of all U chunks are read again together; the abort flag and the time
+        // limit every 8 rounds
+        bool stale = false;
+#pragma unroll
+        for (int u = 0; u < U; ++u)
+#pragma unroll
+            for (int k = 0; k < 4; ++k) stale |= !tag_is(tw[u][k], tag);
+        const uint64_t t0 = stale ? globaltimer_ns() : 0;
+        for (int round = 1; stale; ++round) {
+            __nanosleep(32);
+            stale = false;
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int q = min(q0 + u * CT, chunks - 1);
+                const unsigned long long *w = P.act + ((size_t)(q / cpr) * ld + k0 + (q % cpr) * 8) / 2;
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+                    if (!tag_is(tw[u][k], tag)) {
+                        tw[u][k] = ld_relaxed_u64(w + k);
+                        stale |= !tag_is(tw[u][k], tag);
+                    }
+            }
+            if (stale && (round & 7) == 0 && (aborted(P) || globaltimer_ns() - t0 > WAIT_LIMIT_NS)) {
+                if (!aborted(P)) raise_abort(P, DEV_TIMEOUT_DEP);
+                break;
             }
         }
 #pragma unroll
@@ -408,17 +439,6 @@ __device__ __noinline__ void build_b_act(const MKParams &P, int slice, uint8_t *
             const int q = q0 + u * CT;
             if (q >= chunks) break;
             const int m = q / cpr, c = q % cpr;
-            const unsigned long long *w = P.act + ((size_t)m * ld + k0 + c * 8) / 2;
-            const uint64_t t0 = globaltimer_ns();
-            while (!(tag_is(tw[u][0], tag) && tag_is(tw[u][1], tag) && tag_is(tw[u][2], tag) && tag_is(tw[u][3], tag))) {
-                if (aborted(P) || globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
-                    if (!aborted(P)) raise_abort(P, DEV_TIMEOUT_DEP);
-                    break;
-                }
-                __nanosleep(32);
-                ld_relaxed_2u64(w, tw[u][0], tw[u][1]);
-                ld_relaxed_2u64(w + 2, tw[u][2], tw[u][3]);
-            }
             const int atom = c >> 3, cc = c & 7;
             *reinterpret_cast<uint4 *>(sb + (size_t)atom * P.bn * 128 + m * 128 + ((cc ^ (m & 7)) << 4)) =
                 make_uint4((uint32_t)tw[u][0], (uint32_t)tw[u][1], (uint32_t)tw[u][2], (uint32_t)tw[u][3]);
