@@ -1,8 +1,9 @@
 """Full-size parity on the Qwen3-0.6B shape (28 layers, vocab 151936, rank 16, D = 16).
 
 The oracle runs the 512-token prefill and then three speculative rounds in lockstep with the
-GPU (the GPU verifies the oracle's drafts): logits within 3e-2, draft ids equal up to ties
-inside that tolerance, verify ids, accepted lengths and cached lengths exact.  Properties that
+GPU (the GPU verifies the oracle's drafts): logits within the tolerance below, draft and verify
+ids equal up to ties inside it (both sides continue with the GPU's ids), accepted lengths and
+cached lengths exact.  Properties that
 hold at any size run on the GPU for the whole workloads: speculative output equals plain greedy
 decoding bit for bit, verify rows equal decode rows bit for bit, a sequence's tokens do not
 depend on the batch it shares, and the first greedy tokens match the oracle's."""
@@ -51,10 +52,10 @@ def test_lockstep_rounds_after_512_prefill(big):
     first = eng.pbd_prefill([prompt], max_new=W.max_new)
     cache, p0, lg0 = m.prefill(prompt, P + 8 * (D + 1), want_logits=True)
     cache64, _, _ = m64.prefill(prompt, P + 8 * (D + 1))
+    # the GPU's token is the oracle's argmax up to a tie inside the tolerance; both sides go on
+    # with the GPU's tokens (the prefix cache does not depend on them)
     _check_ids([int(first[0])], lg0[None])
     p = int(first[0])
-    if p != p0:
-        pytest.skip("first token is a near-tie between GPU and oracle; lockstep needs a common start")
     L = P
     for rnd in range(3):
         _, od, _ = m.forward(cache, L, [p] + [-1] * D, True, oracle.MASK_BLOCK_DRAFT, 0, D, want_logits=True)
@@ -65,15 +66,13 @@ def test_lockstep_rounds_after_512_prefill(big):
         assert np.abs(d_lg[0].cpu().numpy() - od).max() <= tol_d
         _check_ids(d_ids[0].cpu().numpy(), od, tol_d)
         drafts = [int(t) for t in np.argmax(od, axis=1)]
-        v_am, ov, _ = m.forward(cache, L, [p] + drafts, False, oracle.MASK_CAUSAL, 0, D + 1, want_logits=True)
+        _, ov, _ = m.forward(cache, L, [p] + drafts, False, oracle.MASK_CAUSAL, 0, D + 1, want_logits=True)
         _, ov64, _ = m64.forward(cache64, L, [p] + drafts, False, oracle.MASK_CAUSAL, 0, D + 1, want_logits=True)
         tol_v = min(0.1, max(TOL, 2 * float(np.abs(ov - ov64).max())))
         v_ids, v_lg = eng.pbd_verify_block(drafts=[drafts], want_logits=True)
         assert np.abs(v_lg[0].cpu().numpy() - ov).max() <= tol_v
         _check_ids(v_ids[0].cpu().numpy(), ov, tol_v)
-        verify = [int(t) for t in v_am]
-        if [int(t) for t in v_ids[0].cpu()] != verify:
-            pytest.skip("verify near-tie in round %d; stop lockstep" % rnd)
+        verify = [int(t) for t in v_ids[0].cpu()]  # checked above against the oracle's logits
         n = oracle.accept_length(drafts, verify)
         n_gpu = eng.pbd_accept_commit()
         assert int(n_gpu[0]) == n
