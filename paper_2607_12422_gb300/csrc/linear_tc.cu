@@ -190,6 +190,199 @@ __global__ void __launch_bounds__(LIN_THREADS, 1)
     if (warp == 0) tmem_dealloc(tmem, LY::TMEM_COLS);
 }
 
+// ------------------------------------------------------------------ persistent lm_head
+//
+// One CTA per SM walks vocabulary tiles t = blockIdx.x, + gridDim.x, ...: the token rows'
+// activation operand (all K atoms) is loaded once and stays in shared memory, weight tiles
+// stream through a ring across tile boundaries, and two TMEM accumulators let the argmax
+// epilogue of one tile run under the MMAs of the next.  Warp 0 streams, warp 1 issues the
+// MMAs, warps 2-5 (one per TMEM lane quarter) reduce each token row's (max, argmax) over the
+// tile's 128 vocabulary rows, lowest index on ties, as k_linear_tc<BN, EPI_ARGMAX> does.
+constexpr int LMH_THREADS = 192;
+constexpr int LMH_STAGES = 4;
+
+template <int BN>
+struct LmhLayout {
+    static constexpr int X_ATOM = BN * 128;  // one 64-wide K atom of the token rows
+    static constexpr int RING_OFF = 0;
+    static constexpr int X_OFF = LMH_STAGES * TILE_BYTES;
+    static constexpr int MAX_ATOMS = 16;     // K <= 1024
+    static constexpr int BAR_OFF = X_OFF + MAX_ATOMS * X_ATOM;
+    static constexpr int RED_OFF = BAR_OFF + 256;
+    static constexpr int RED_BYTES = 2 * 4 * BN * 8;  // [acc][quarter][token] (value, index)
+    static constexpr int TOTAL = RED_OFF + RED_BYTES + 1024;
+    static constexpr uint32_t TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;
+};
+
+template <int BN>
+__global__ void __launch_bounds__(LMH_THREADS, 1)
+    k_lm_head(const __grid_constant__ CUtensorMap xmap, const uint8_t *__restrict__ wtiles, int k_tiles, int n_tiles,
+              int M, float *__restrict__ tile_max, int *__restrict__ tile_arg, float *__restrict__ logits, int V,
+              int *status) {
+    using LY = LmhLayout<BN>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *ring = base + LY::RING_OFF;
+    uint8_t *sx = base + LY::X_OFF;
+    uint64_t *full = reinterpret_cast<uint64_t *>(base + LY::BAR_OFF);
+    uint64_t *empty = full + LMH_STAGES;
+    uint64_t *x_full = empty + LMH_STAGES;
+    uint64_t *acc_full = x_full + 1;   // [2]
+    uint64_t *acc_empty = acc_full + 2;  // [2]
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_empty + 2);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+    float *red_val = reinterpret_cast<float *>(base + LY::RED_OFF);
+    int *red_idx = reinterpret_cast<int *>(red_val + 2 * 4 * BN);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n_my = blockIdx.x < n_tiles ? (n_tiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < LMH_STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(x_full, 1);
+        mbar_init(&acc_full[0], 1);
+        mbar_init(&acc_full[1], 1);
+        mbar_init(&acc_empty[0], 1);
+        mbar_init(&acc_empty[1], 1);
+        *abort_flag = 0;
+        fence_mbarrier_init();
+        prefetch_tensormap(&xmap);
+    }
+    if (warp == 0) tmem_alloc(tmem_slot, LY::TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0 && lane == 0) {
+        // ---- producer: the token rows once, then the CTA's weight tiles back to back
+        mbar_arrive_expect_tx(x_full, (uint32_t)(k_tiles * LY::X_ATOM));
+        for (int a = 0; a < k_tiles; ++a) tma_load_2d(sx + a * LY::X_ATOM, &xmap, a * KT, 0, x_full);
+        const uint64_t pol = l2_policy_evict_first();
+        int g = 0;
+        for (int j = 0; j < n_my && !*abort_flag; ++j) {
+            const uint8_t *wsrc = wtiles + (size_t)(blockIdx.x + j * gridDim.x) * k_tiles * TILE_BYTES;
+            for (int s = 0; s < k_tiles; ++s, ++g) {
+                const int slot = g % LMH_STAGES;
+                if (g >= LMH_STAGES &&
+                    !mbar_wait(&empty[slot], ((g / LMH_STAGES) - 1) & 1, status, DEV_TIMEOUT_SLOT, abort_flag))
+                    break;
+                mbar_arrive_expect_tx(&full[slot], (uint32_t)TILE_BYTES);
+                bulk_g2s(ring + slot * TILE_BYTES, wsrc + (size_t)s * TILE_BYTES, TILE_BYTES, &full[slot], pol);
+            }
+        }
+        if (*abort_flag) {
+            // error path: give the copies still in flight a bounded chance to land before exit
+            mbar_wait(x_full, 0, nullptr, 0, nullptr);
+            for (int h = g > LMH_STAGES ? g - LMH_STAGES : 0; h < g; ++h)
+                mbar_wait(&full[h % LMH_STAGES], (h / LMH_STAGES) & 1, nullptr, 0, nullptr);
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---- MMA issuer: per tile 4 x (128 x BN x 16) per K atom into accumulator j & 1
+        const uint32_t idesc = idesc_bf16_f32(128, BN);
+        bool ok = mbar_wait(x_full, 0, status, DEV_TIMEOUT_LOAD, abort_flag);
+        tc_fence_after();
+        int g = 0;
+        for (int j = 0; ok && j < n_my; ++j) {
+            const int acc = j & 1;
+            if (j >= 2 && !mbar_wait(&acc_empty[acc], ((j >> 1) - 1) & 1, status, DEV_TIMEOUT_MMA, abort_flag)) break;
+            tc_fence_after();
+            const uint32_t d = tmem + (uint32_t)(acc * BN);
+            for (int s = 0; s < k_tiles; ++s, ++g) {
+                const int slot = g % LMH_STAGES;
+                if (!mbar_wait(&full[slot], (g / LMH_STAGES) & 1, status, DEV_TIMEOUT_LOAD, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint64_t ad = sw128_kmajor_desc(ring + slot * TILE_BYTES);
+                const uint64_t bd = sw128_kmajor_desc(sx + s * LY::X_ATOM);
+#pragma unroll
+                for (int kk = 0; kk < KT / 16; ++kk)
+                    mma_bf16_ss(d, ad + 2ull * kk, bd + 2ull * kk, idesc, (s | kk) != 0 ? 1u : 0u);
+                mma_commit(&empty[slot]);
+            }
+            if (ok) mma_commit(&acc_full[acc]);
+        }
+    } else if (warp >= 2) {
+        // ---- epilogue: warp w reads TMEM lane quarter w % 4 (32 vocabulary rows)
+        const int q = warp & 3;
+        const int row = q * 32 + lane;
+        for (int j = 0; j < n_my; ++j) {
+            const int acc = j & 1, tile = blockIdx.x + j * gridDim.x;
+            if (!mbar_wait(&acc_full[acc], (j >> 1) & 1, status, DEV_TIMEOUT_MMA, abort_flag)) break;
+            tc_fence_after();
+            const int feat = tile * TILE_ROWS + row;
+            float *rv = red_val + acc * 4 * BN;
+            int *ri = red_idx + acc * 4 * BN;
+            for (int c0 = 0; c0 < BN && c0 < M; c0 += 32) {
+                uint32_t v[32];
+                tmem_ld_32cols(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN + c0), v);
+                tmem_ld_wait();
+#pragma unroll
+                for (int jj = 0; jj < 32; ++jj) {
+                    const int tok = c0 + jj;
+                    if (tok >= M) break;  // uniform across the warp
+                    float bv = __uint_as_float(v[jj]);
+                    int bi = feat;
+                    if (logits != nullptr) logits[(size_t)tok * V + feat] = bv;
+#pragma unroll
+                    for (int off = 16; off >= 1; off >>= 1) {
+                        const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+                        const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+                        if (ov > bv || (ov == bv && oi < bi)) {
+                            bv = ov;
+                            bi = oi;
+                        }
+                    }
+                    if (lane == 0) {
+                        rv[q * BN + tok] = bv;
+                        ri[q * BN + tok] = bi;
+                    }
+                }
+            }
+            tc_fence_before();
+            asm volatile("bar.sync 1, 128;" ::: "memory");  // the four epilogue warps
+            if (warp == 2) {
+                for (int c = lane; c < M; c += 32) {
+                    float bv = rv[c];
+                    int bi = ri[c];
+#pragma unroll
+                    for (int w = 1; w < 4; ++w) {
+                        const float ov = rv[w * BN + c];
+                        const int oi = ri[w * BN + c];
+                        if (ov > bv || (ov == bv && oi < bi)) {
+                            bv = ov;
+                            bi = oi;
+                        }
+                    }
+                    tile_max[(size_t)tile * M + c] = bv;
+                    tile_arg[(size_t)tile * M + c] = bi;
+                }
+                __syncwarp();
+                // the accumulator and this tile's reduction slots may be reused
+                if (lane == 0) mbarrier_arrive_one(&acc_empty[acc]);
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, LY::TMEM_COLS);
+}
+
+static int lm_head_grid() {
+    static int sms = 0;
+    if (sms == 0) {
+        int dev = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+            sms = 0;
+    }
+    return sms;
+}
+
 template <int BN, int EPI>
 static cudaError_t configure_one() {
     return cudaFuncSetAttribute(k_linear_tc<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -205,7 +398,11 @@ cudaError_t configure_linear_kernels() {
     if ((e = configure_one<32, EPI_ARGMAX>()) != cudaSuccess) return e;
     if ((e = configure_one<64, EPI_ARGMAX>()) != cudaSuccess) return e;
     if ((e = configure_one<128, EPI_ARGMAX>()) != cudaSuccess) return e;
-    return configure_one<256, EPI_ARGMAX>();
+    if ((e = configure_one<256, EPI_ARGMAX>()) != cudaSuccess) return e;
+    if ((e = cudaFuncSetAttribute(k_lm_head<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, LmhLayout<32>::TOTAL)) !=
+        cudaSuccess)
+        return e;
+    return cudaFuncSetAttribute(k_lm_head<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, LmhLayout<64>::TOTAL);
 }
 
 template <int BN, int EPI>
@@ -239,6 +436,20 @@ cudaError_t launch_linear_partials(const CUtensorMap *x_map, int bn, const Tiled
 cudaError_t launch_lm_head(const CUtensorMap *x_map, int bn, const TiledWeight &w, int M, float *tile_max,
                            int *tile_arg, float *logits, int *status, cudaStream_t st) {
     const int n_tiles = w.n_main / TILE_ROWS;
+    const int k_tiles = w.K / KT;
+    const int grid = std::min(lm_head_grid(), n_tiles);
+    // a few token rows: the persistent kernel (operand resident, one CTA per SM)
+    if ((bn == 32 || bn == 64) && k_tiles <= LmhLayout<32>::MAX_ATOMS && grid > 0) {
+        if (bn == 32)
+            k_lm_head<32><<<grid, LMH_THREADS, LmhLayout<32>::TOTAL, st>>>(
+                *x_map, static_cast<const uint8_t *>(w.tiles), k_tiles, n_tiles, M, tile_max, tile_arg, logits, w.n_main,
+                status);
+        else
+            k_lm_head<64><<<grid, LMH_THREADS, LmhLayout<64>::TOTAL, st>>>(
+                *x_map, static_cast<const uint8_t *>(w.tiles), k_tiles, n_tiles, M, tile_max, tile_arg, logits, w.n_main,
+                status);
+        return cudaGetLastError();
+    }
     switch (bn) {
         case 32: return launch_tc<32, EPI_ARGMAX>(x_map, w, n_tiles, 1, M, nullptr, 0, 0, tile_max, tile_arg, logits,
                                                   status, st);
