@@ -208,6 +208,94 @@ def main_reference(args):
     return 0
 
 
+def run_rounds(e, prompts, G, D, mode, steps, warmup, forced=None):
+    """`warmup` then `steps` timed rounds over generations of `prompts` on engine e.  A chunk never
+    holds more rounds than the budget left could absorb at full acceptance (for the sequence
+    furthest along), so no timed round runs past a finished generation; the prompts are prefilled
+    again (untimed) when the budget is spent.  Returns (per-phase ms sums, tokens emitted in timed
+    rounds over all sequences, kernel launches, mean cached length summed over sequences).
+    forced: [rounds, batch] accepted lengths, consumed in order across the calls."""
+    acc = np.zeros(4)
+    f_off = 0
+
+    def chunk_forced(k):
+        nonlocal f_off
+        if forced is None:
+            return None
+        idx = (f_off + np.arange(k)) % len(forced)
+        f_off += k
+        return np.ascontiguousarray(forced[idx])
+    tokens = 0
+    launches = 0
+    l_sum = 0.0
+    per_round = (D + 1) if mode == 0 else 1
+    e.pbd_prefill(prompts, max_new=G)
+    done_w, left = 0, steps
+    while done_w < warmup or left > 0:
+        L0, _, n0 = e.pbd_get_state()
+        room = (G - int(np.max(n0[:len(prompts)]))) // per_round
+        if room < 1:
+            e.pbd_prefill(prompts, max_new=G)
+            continue
+        if done_w < warmup:
+            k = min(warmup - done_w, room, CHUNK)
+            e.pbd_bench_rounds(mode, 0, k, chunk_forced(k))
+            done_w += k
+            continue
+        k = min(left, room, CHUNK)
+        r = e.pbd_bench_rounds(mode, 0, k, chunk_forced(k))
+        L1, _, n1 = e.pbd_get_state()
+        acc += np.array(r[:4])
+        tokens += int(np.sum(n1[:len(prompts)])) - int(np.sum(n0[:len(prompts)]))
+        launches += r[4] * k
+        l_sum += 0.5 * (int(np.sum(L0[:len(prompts)])) + int(np.sum(L1[:len(prompts)]))) * k
+        left -= k
+    return acc, tokens, launches, l_sum / steps
+
+
+def measure_configs(pbd, synth, base, ad, dev, hbm, warmup):
+    """The other workloads of the 0.6B shape: a 4096-token prompt, a batch of 8 ragged prompts,
+    and the block-size sweep with forced acceptance (means 1, 3, 6) beside plain decoding."""
+    out = {}
+    for name, steps in (("qwen3-0.6b-b1-d16-p4096-g512", 48), ("qwen3-0.6b-b8-d16-p256to2048-g256", 32)):
+        W = synth.WORKLOADS[name]
+        S, D = W.shape, W.block_D
+        prompts = synth.gen_prompts(S, list(W.prompt_lens))
+        e = pbd.Engine(S, base, ad, block_D=D, max_batch=len(prompts), max_seq_len=max(W.prompt_lens) + W.max_new + 8,
+                       device=dev)
+        acc, tok, _, L_sum = run_rounds(e, prompts, W.max_new, D, 0, steps, warmup)
+        e.close()
+        d_us, v_us = 1e3 * acc[0] / steps, 1e3 * acc[1] / steps
+        B = len(prompts)
+        # one verify pass of the batch: every weight once, each sequence's KV once, B (D+1) rows written
+        fl_v = pass_bytes(S, L_sum, B * (D + 1), False) / (hbm * 1e9) * 1e6
+        out[name] = {"batch": B, "draft_us": d_us, "verify_us": v_us, "tokens_per_s": tok / (acc[3] / 1e3),
+                     "mean_tokens_per_round_per_seq": tok / steps / B, "kv_tokens_mean": L_sum,
+                     "verify_roofline_frac": fl_v / v_us, "steps": steps}
+    W = synth.WORKLOADS["qwen3-0.6b-b1-p1024-dsweep-forced"]
+    S = W.shape
+    prompt = synth.gen_prompts(S, list(W.prompt_lens))
+    sweep = {}
+    for D in W.D_sweep:
+        e = pbd.Engine(S, base, ad, block_D=D, max_batch=1, max_seq_len=W.prompt_lens[0] + W.max_new + 2 * D + 8,
+                       device=dev)
+        acc_ar, tok_ar, _, _ = run_rounds(e, prompt, W.max_new, D, 1, 32, warmup)
+        ar_us = 1e3 * acc_ar[3] / 32
+        row = {"ar_us_per_token": ar_us}
+        for mean in W.forced_means:
+            steps = 48
+            forced = synth.forced_accept_lengths(mean, D, steps + warmup).reshape(-1, 1)
+            acc, tok, _, _ = run_rounds(e, prompt, W.max_new, D, 0, steps, warmup, forced)
+            step_us = 1e3 * acc[3] / steps
+            row["mean_A_%g" % mean] = {"step_us": step_us, "tokens_per_s": tok / (acc[3] / 1e3),
+                                       "tokens_per_round": tok / steps, "speedup_vs_ar": (tok / steps) * ar_us / step_us}
+        row["break_even_accept"] = (1e3 * acc[0] / steps + 1e3 * acc[1] / steps) / ar_us
+        e.close()
+        sweep["D=%d" % D] = row
+    out[W.name] = sweep
+    return out
+
+
 def main(args):
     ws, rank, local = dist_setup(args)
     import torch
@@ -226,39 +314,7 @@ def main(args):
     eng = pbd.Engine(S, base, ad, block_D=D, max_batch=1, max_seq_len=P + G + 8, device=dev)
 
     def timed_rounds(mode, steps, warmup, forced=None, e=None):
-        """`warmup` then `steps` timed rounds over generations of the workload (on engine e,
-        default the main one).  A chunk never holds
-        more rounds than the budget left could absorb at full acceptance, so no timed round runs
-        past a finished generation; a new prompt is prefilled (untimed) when the budget is spent.
-        Returns (per-phase ms sums, tokens emitted in timed rounds, kernel launches, mean L)."""
-        e = e or eng
-        acc = np.zeros(4)
-        tokens = 0
-        launches = 0
-        l_sum = 0.0
-        per_round = (D + 1) if mode == 0 else 1
-        e.pbd_prefill([prompt], max_new=G)
-        done_w, left = 0, steps
-        while done_w < warmup or left > 0:
-            L0, _, n0 = e.pbd_get_state()
-            room = (G - int(n0[0])) // per_round
-            if room < 1:
-                e.pbd_prefill([prompt], max_new=G)
-                continue
-            if done_w < warmup:
-                k = min(warmup - done_w, room, CHUNK)
-                e.pbd_bench_rounds(mode, 0, k, forced)
-                done_w += k
-                continue
-            k = min(left, room, CHUNK)
-            r = e.pbd_bench_rounds(mode, 0, k, forced)
-            L1, _, n1 = e.pbd_get_state()
-            acc += np.array(r[:4])
-            tokens += int(n1[0]) - int(n0[0])
-            launches += r[4] * k
-            l_sum += 0.5 * (int(L0[0]) + int(L1[0])) * k
-            left -= k
-        return acc, tokens, launches, l_sum / steps
+        return run_rounds(e or eng, [prompt], G, D, mode, steps, warmup, forced)
 
     hbm, peak_kind = peaks()
     if args.profile_rounds:
@@ -345,6 +401,10 @@ def main(args):
             ev.close()
             del ev
 
+    configs = None
+    if ws == 1 and not args.no_configs:
+        configs = measure_configs(pbd, synth, base, ad, dev, hbm, args.warmup)
+
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         tps, sec, done, threads = run_cpu_oracle(S, base, ad, 64, D, 24, max_seconds=20)
@@ -369,6 +429,7 @@ def main(args):
             "ar": {"us_per_step": ar_us, "pass_us": ar_pass_us, "tokens_per_s": tok_ar / (acc_ar[3] / 1e3),
                    "break_even_accept": (draft_us + verify_us) / ar_us},
             "draft_variants": variants,
+            "other_workloads": configs,
             "roofline": {"bound": "hbm", "kernel": "k_pass (persistent; 28 layers of one verify pass, 17 rows)",
                          "achieved": achieved, "peak": hbm, "peak_kind": peak_kind + " hbm_gbs (burst)",
                          "unit": "GB/s", "frac": achieved / hbm, "traffic": traffic,
@@ -398,6 +459,7 @@ if __name__ == "__main__":
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-variants", action="store_true", help="skip the draft-variant measurements")
+    ap.add_argument("--no-configs", action="store_true", help="skip the long-context, batch-8 and D-sweep workloads")
     ap.add_argument("--profile-rounds", action="store_true",
                     help="only prefill + warm-up + timed rounds (the configuration profiled under ncu)")
     a = ap.parse_args()
