@@ -850,9 +850,13 @@ __device__ __noinline__ void attn_combine(const MKParams &P, int bl, int g, int 
 #pragma unroll
         for (int u = 0; u < NB; ++u)
             if (v[u].y > 0.f) mx = fmaxf(mx, v[u].x);
-        for (int s0 = NB; s0 < nv; ++s0) {  // long contexts only
-            const float2 w = __ldcg(ml + s0);
-            if (w.y > 0.f) mx = fmaxf(mx, w.x);
+        for (int s0 = NB; s0 < nv; s0 += NB) {  // long contexts only: NB statistics per round
+            float2 w[NB];
+#pragma unroll
+            for (int u = 0; u < NB; ++u) w[u] = s0 + u < nv ? __ldcg(ml + s0 + u) : make_float2(-INFINITY, 0.f);
+#pragma unroll
+            for (int u = 0; u < NB; ++u)
+                if (w[u].y > 0.f) mx = fmaxf(mx, w[u].x);
         }
         float num[E];
 #pragma unroll
