@@ -112,13 +112,24 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+def source_hash(path):
+    """Hash of a CUDA source with its comments and blank space removed: a comment edit leaves the
+    compiled kernel, and therefore its measured traffic, unchanged."""
+    import re
+    txt = open(path).read()
+    txt = re.sub(r"//[^\n]*", "", re.sub(r"/\*.*?\*/", "", txt, flags=re.S))
+    txt = re.sub(r"\s+", " ", txt).strip()
+    return hashlib.sha256(txt.encode()).hexdigest()[:16]
+
+
 def traffic_for(kernel_src):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel source is unchanged since."""
+    """DRAM bytes per launch from the committed ncu summary, if the kernel source is unchanged since
+    (comments aside)."""
     path = os.path.join(ROOT, "profiles", "k_pass_verify_qwen3_0.6b_traffic.json")
     try:
         with open(path) as f:
             rec = json.load(f)
-        h = hashlib.sha256(open(kernel_src, "rb").read()).hexdigest()[:16]
+        h = source_hash(kernel_src)
         if rec.get("source_sha256_16") == h:
             return float(rec["dram_bytes_per_launch"])
     except Exception:

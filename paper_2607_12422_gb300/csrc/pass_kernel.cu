@@ -4,8 +4,8 @@
 // Why: at batch 1 and D = 16 a pass moves 1.2 GB of weights (~180 us at full HBM bandwidth)
 // through ~500 small dependent steps.  As separate kernel launches, launch gaps and latency
 // chains dominated.  Here one CTA per SM walks a static, topologically ordered list of work
-// items, and items wait only for the items they read (per-tile counters in global memory with
-// bounded spins), so phases overlap and no kernel boundary separates them.
+// items, and items wait only for the items they read (completion counters or tagged words in
+// global memory, with bounded spins), so phases overlap and no kernel boundary separates them.
 //
 // Roles inside a CTA (256 threads):
 //   warp 0      weight producer: walks the CTA's linear items ahead of the others and streams
@@ -29,7 +29,8 @@
 //   down tile    -> + adapter delta, residual add into h, per-tile sum of squares of h
 // The adapter's A rows form one extra tile whose partials u = x A^T the reducers above sum
 // themselves.  Each reduction then counts once, with release semantics, on the counter its
-// consumers poll (attention inputs per KV head, a down-projection K slice, the residual).
+// consumers poll (attention inputs per KV head, the residual), except gate|up: SiLU(gate) * up
+// goes out as tagged words that the down projection's operand staging polls.
 // Attention items cover (sequence, KV head, 128-key split); when the splits sit on distinct
 // CTAs they wait for one another and each merges a share of the rows, else the last one
 // merges all.  RMSNorm statistics are summed per 128-feature
