@@ -198,6 +198,15 @@ pbd_status pbd_time_pass(pbd_ctx *ctx, int32_t kind, int32_t iters, double *h_ms
 pbd_status pbd_trace_pass(pbd_ctx *ctx, int32_t kind, int32_t *h_items, uint64_t *h_trace, int32_t cap,
                           int32_t *h_n);
 
+/* Failure-detection check (no GPU fault is involved).  On a prefilled context, runs one verify
+ * pass whose schedule lacks the first q|k|v item of layer 0: that item's partial sums never
+ * arrive, so the waits polling for them run out after their bound (1 s), latch a device code
+ * and end the pass.  Returns PBD_ERR_DEVICE with the latched code in *h_device_code (a
+ * DEV_TIMEOUT_* value; 0 would mean the pass ended without noticing).  The cached tokens and
+ * the decoding state are untouched (the pass writes scratch slots only) and the context stays
+ * usable: the normal schedules are restored before returning.  Synchronous. */
+pbd_status pbd_check_stalled_pass(pbd_ctx *ctx, int32_t *h_device_code);
+
 const char *pbd_last_error(const pbd_ctx *ctx);
 
 /* Build/version tag of the library ("pbd sm_103a <date>"). */

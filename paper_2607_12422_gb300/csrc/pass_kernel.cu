@@ -153,6 +153,15 @@ __device__ bool spin_until(const int *c, int target, const MKParams &P) {
     }
 }
 
+// bounded mbarrier wait that does not give up on abort: the pass is ending and its asynchronous
+// copies and MMAs must land before the CTA releases its shared memory and TMEM
+__device__ __forceinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
+    const uint32_t a = smem_u32(bar);
+    const uint64_t t0 = globaltimer_ns();
+    while (!mbar_try_wait(a, parity) && globaltimer_ns() - t0 < WAIT_LIMIT_NS) {
+    }
+}
+
 // bounded mbarrier wait that also gives up when the pass is aborted
 __device__ bool mbar_wait_mk(uint64_t *bar, uint32_t parity, const MKParams &P, int code) {
     const uint32_t a = smem_u32(bar);
@@ -960,7 +969,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *ring = base;
     uint8_t *uni = base + P.ring_bytes;  // activation tile / attention staging
-    __shared__ __align__(8) uint64_t full[MAX_SLOT], empty[MAX_SLOT], b_full[2], b_empty, acc_full, att_bar;
+    __shared__ __align__(8) uint64_t full[MAX_SLOT], empty[MAX_SLOT], b_full[2], b_empty, acc_full, att_bar, mma_drain;
     __shared__ uint32_t tmem_slot;
     // compute-group flags: each is written by thread 0 and read by all after a barrier, and is
     // not written again before every thread has passed at least one more barrier
@@ -987,6 +996,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
         mbar_init(&b_empty, 1);
         mbar_init(&acc_full, 1);
         mbar_init(&att_bar, 1);
+        mbar_init(&mma_drain, 1);
         prefetch_tensormap(&P.kmap);
         prefetch_tensormap(&P.vmap);
         fence_mbarrier_init();
@@ -1029,6 +1039,9 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 }
                 if (!ok) break;
             }
+            if (aborted(P))  // the last nslot tiles issued may still be in flight: let them land
+                for (uint32_t h = kt > (uint32_t)P.nslot ? kt - P.nslot : 0; h < kt; ++h)
+                    drain_wait(&full[h % P.nslot], (h / P.nslot) & 1);
         }
     } else if (warp == 1) {
         // ---------------- MMA issuer
@@ -1071,6 +1084,11 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 mma_commit(&acc_full);
                 ++li;
                 if (na > HALF_ATOMS) ++l8;
+            }
+            if (aborted(P)) {
+                // every MMA issued so far completes before TMEM and the operands are released
+                mma_commit(&mma_drain);
+                drain_wait(&mma_drain, 0);
             }
         }
     } else {

@@ -1010,6 +1010,44 @@ pbd_status pbd_time_pass(pbd_ctx *c, int32_t kind, int32_t iters, double *h_ms_p
     return check_device(c);
 }
 
+pbd_status pbd_check_stalled_pass(pbd_ctx *c, int32_t *h_device_code) {
+    if (!c || !h_device_code) return fail(c, PBD_ERR_INVALID_ARG, "null argument");
+    if (c->phase != PH_READY) return fail(c, PBD_ERR_STATE, "the check needs a prefilled or committed state");
+    const PassDesc pd = block_pass(c, PK_VERIFY);
+    const std::vector<int> ns = decode_splits(c);
+    std::vector<MKItem> all, items;
+    std::vector<int> off;
+    mk_build_schedule(c->dm, pd, ns, 1, &all, &off);  // one CTA: the items in order
+    bool dropped = false;
+    for (const MKItem &it : all) {
+        if (!dropped && it.op == MK_LINEAR && it.lin == 0 && it.layer == 0) {
+            dropped = true;
+            continue;
+        }
+        items.push_back(it);
+    }
+    // deal the remaining items round-robin, as mk_build_schedule does
+    std::vector<int> cta_off(c->grid + 1, 0);
+    for (size_t i = 0; i < items.size(); ++i) cta_off[i % c->grid + 1]++;
+    for (int k = 0; k < c->grid; ++k) cta_off[k + 1] += cta_off[k];
+    std::vector<MKItem> dealt(items.size());
+    std::vector<int> fill(cta_off.begin(), cta_off.end() - 1);
+    for (size_t i = 0; i < items.size(); ++i) dealt[fill[i % c->grid]++] = items[i];
+    Sched &sv = c->sched[PK_VERIFY];
+    CK(cudaMemcpyAsync(sv.items, dealt.data(), dealt.size() * sizeof(MKItem), cudaMemcpyHostToDevice, c->st));
+    CK(cudaMemcpyAsync(sv.off, cta_off.data(), cta_off.size() * sizeof(int), cudaMemcpyHostToDevice, c->st));
+    CK(cudaStreamSynchronize(c->st));
+    CK(launch_build_ids(pd, 1, c->s.pending, c->draft_ids, c->D, c->ids, c->st));
+    TRY(enqueue_pass_kernel(c, pd, PK_VERIFY));
+    CK(cudaStreamSynchronize(c->st));
+    int code = 0;
+    CK(cudaMemcpy(&code, c->status, sizeof(int), cudaMemcpyDeviceToHost));
+    *h_device_code = code;
+    // the normal verify schedule again; the device code is reported (and cleared) below
+    TRY(upload_schedule(c, PK_VERIFY, pd, ns));
+    return check_device(c);
+}
+
 pbd_status pbd_trace_pass(pbd_ctx *c, int32_t kind, int32_t *h_items, uint64_t *h_trace, int32_t cap, int32_t *h_n) {
     if (!c || !h_items || !h_trace || !h_n) return fail(c, PBD_ERR_INVALID_ARG, "null argument");
     if (kind < 0 || kind > 2) return fail(c, PBD_ERR_INVALID_ARG, "kind in [0,2]");

@@ -97,6 +97,8 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     L.pbd_trace_pass.restype = C.c_int
     L.pbd_bench_rounds.restype = C.c_int
     L.pbd_time_pass.restype = C.c_int
+    L.pbd_check_stalled_pass.argtypes = [P, P]
+    L.pbd_check_stalled_pass.restype = C.c_int
     L.pbd_op_linear_workspace_bytes.restype = C.c_size_t
     L.pbd_op_linear_workspace_bytes.argtypes = [I32, I32, I32, I32]
     L.pbd_op_linear.argtypes = [I32, I32, I32, I32, C.c_float, P, P, P, P, P, P, C.c_size_t, P]
@@ -381,6 +383,12 @@ class Engine:
         self._call(self.lib.pbd_trace_pass, kind, items.ctypes.data, tr.ctypes.data, cap, n.ctypes.data)
         k = int(n[0])
         return items[: 4 * k].reshape(k, 4), tr[: 8 * k].reshape(k, 8)
+
+    def pbd_check_stalled_pass(self):
+        """(status, device code) of a verify pass missing one item (see include/pbd.h)."""
+        code = np.zeros(1, np.int32)
+        status = self.lib.pbd_check_stalled_pass(self.ctx, code.ctypes.data)
+        return int(status), int(code[0])
 
     def pbd_time_pass(self, kind: int, iters: int):
         """(ms per launch, algorithmic bytes per launch) of the persistent pass kernel timed alone

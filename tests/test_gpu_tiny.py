@@ -223,3 +223,20 @@ def test_pass_timing_and_trace_entry_points(env):
     # the context is still in the state a round starts from
     d1, _ = eng.pbd_draft_block()
     assert d1.shape == (1, D)
+
+
+def test_stalled_pass_is_reported_and_context_survives(env):
+    """Failure detection without a GPU fault: a verify pass whose schedule lacks one q|k|v item
+    never receives that item's partial sums; the bounded waits run out (about a second), the
+    device code is latched and reported as PBD_ERR_DEVICE, the decoding state is untouched and
+    the context keeps decoding exactly."""
+    eng, m, prompt = env["eng"], env["model"], env["prompts"][0]
+    P = len(prompt)
+    eng.pbd_prefill([prompt], max_new=32)
+    status, code = eng.pbd_check_stalled_pass()
+    assert status == 6  # PBD_ERR_DEVICE
+    assert code in (1, 2, 3, 6)  # a DEV_TIMEOUT_* code
+    L, pend, n_out = eng.pbd_get_state()
+    assert int(L[0]) == P and int(n_out[0]) == 1
+    out, st = eng.pbd_generate([prompt], 32, mode=0)
+    assert [int(t) for t in out[0].cpu()] == oracle.greedy_generate(m, prompt, 32)
