@@ -207,6 +207,20 @@ pbd_status pbd_trace_pass(pbd_ctx *ctx, int32_t kind, int32_t *h_items, uint64_t
  * usable: the normal schedules are restored before returning.  Synchronous. */
 pbd_status pbd_check_stalled_pass(pbd_ctx *ctx, int32_t *h_device_code);
 
+/* The work schedule of one pass, computed on the host with no context and no GPU (for checks
+ * of the schedule's properties).  For a generation of `batch` prompts of h_prompt_lens tokens
+ * and a budget of max_new tokens under cfg (whose draft variant applies to kind 0), returns the
+ * items of a draft (kind 0), verify (1) or plain-decoding (2) pass dealt round-robin over `grid`
+ * CTAs: h_items[4 i..4 i+3] = {op | lin << 8 | layer << 16, a, b, c} (op 0 embedding row, 1
+ * linear slice, 2 attention split, 3 final norm; see pbd_trace_pass), grouped by CTA with CTA
+ * k's items at [h_cta_off[k], h_cta_off[k + 1]) (h_cta_off has grid + 1 entries; CTA k takes
+ * the topologically ordered list's items k, k + grid, ...).  *h_n is the item count; at most
+ * `cap` items are written (PBD_ERR_CAPACITY beyond).  Errors: PBD_ERR_INVALID_ARG (bad config or
+ * argument), PBD_ERR_CAPACITY (prompt plus budget beyond max_seq_len, or cap too small). */
+pbd_status pbd_plan_pass(const pbd_config *cfg, int32_t kind, int32_t batch, const int32_t *h_prompt_lens,
+                         int32_t max_new, int32_t grid, int32_t *h_items, int32_t *h_cta_off, int32_t cap,
+                         int32_t *h_n);
+
 const char *pbd_last_error(const pbd_ctx *ctx);
 
 /* Build/version tag of the library ("pbd sm_103a <date>"). */

@@ -595,6 +595,41 @@ size_t pbd_workspace_bytes(const pbd_config *cfg) {
     return layout(&tmp, nullptr);
 }
 
+pbd_status pbd_plan_pass(const pbd_config *cfg, int32_t kind, int32_t batch, const int32_t *h_prompt_lens,
+                         int32_t max_new, int32_t grid, int32_t *h_items, int32_t *h_cta_off, int32_t cap, int32_t *h_n) {
+    std::string why;
+    if (!valid_config(cfg, &why)) return fail(nullptr, PBD_ERR_INVALID_ARG, "%s", why.c_str());
+    if (kind < 0 || kind > 2 || batch < 1 || batch > cfg->max_batch || !h_prompt_lens || max_new < 1 || grid < 1 ||
+        !h_items || !h_cta_off || !h_n)
+        return fail(nullptr, PBD_ERR_INVALID_ARG, "pbd_plan_pass: bad argument");
+    for (int b = 0; b < batch; ++b)
+        if (h_prompt_lens[b] < 1 || h_prompt_lens[b] + max_new > cfg->max_seq_len)
+            return fail(nullptr, PBD_ERR_CAPACITY, "prompt %d of %d tokens + %d exceeds max_seq_len", b,
+                        h_prompt_lens[b], max_new);
+    pbd_ctx tmp;
+    tmp.cfg = *cfg;
+    tmp.dm = Dims{cfg->n_layers, cfg->hidden,      cfg->n_q_heads, cfg->n_kv_heads, cfg->head_dim,
+                  cfg->intermediate, cfg->vocab, cfg->lora_rank, cfg->rms_eps,     cfg->lora_scale};
+    tmp.grid = grid;
+    layout(&tmp, nullptr);
+    tmp.batch = batch;
+    tmp.max_new = max_new;
+    tmp.prompt_lens.assign(h_prompt_lens, h_prompt_lens + batch);
+    std::vector<MKItem> items;
+    std::vector<int> off;
+    mk_build_schedule(tmp.dm, block_pass(&tmp, kind), decode_splits(&tmp), grid, &items, &off);
+    *h_n = (int32_t)items.size();
+    if ((int)items.size() > cap) return fail(nullptr, PBD_ERR_CAPACITY, "%zu items exceed cap %d", items.size(), cap);
+    for (size_t i = 0; i < items.size(); ++i) {
+        h_items[4 * i] = items[i].op | (items[i].lin << 8) | (items[i].layer << 16);
+        h_items[4 * i + 1] = items[i].a;
+        h_items[4 * i + 2] = items[i].b;
+        h_items[4 * i + 3] = items[i].c;
+    }
+    for (int k = 0; k <= grid; ++k) h_cta_off[k] = off[k];
+    return PBD_OK;
+}
+
 pbd_status pbd_create(const pbd_config *cfg, const pbd_base_weights *base, const pbd_adapter_weights *adapter,
                       void *d_workspace, size_t workspace_bytes, void *d_stream, pbd_ctx **out) {
     pbd_ctx *c = nullptr;

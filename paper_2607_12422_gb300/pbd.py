@@ -99,6 +99,8 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     L.pbd_time_pass.restype = C.c_int
     L.pbd_check_stalled_pass.argtypes = [P, P]
     L.pbd_check_stalled_pass.restype = C.c_int
+    L.pbd_plan_pass.argtypes = [C.POINTER(pbd_config), I32, I32, P, I32, I32, P, P, I32, P]
+    L.pbd_plan_pass.restype = C.c_int
     L.pbd_op_linear_workspace_bytes.restype = C.c_size_t
     L.pbd_op_linear_workspace_bytes.argtypes = [I32, I32, I32, I32]
     L.pbd_op_linear.argtypes = [I32, I32, I32, I32, C.c_float, P, P, P, P, P, P, C.c_size_t, P]
@@ -193,6 +195,21 @@ def make_config(shape, block_D: int, max_batch: int, max_seq_len: int, draft_lay
                       shape.intermediate, shape.vocab, shape.rms_eps, shape.rope_theta, shape.lora_rank,
                       shape.lora_alpha / shape.lora_rank, block_D, max_batch, max_seq_len, 16,
                       draft_layers, denoise_steps, 0 if anchored else 1)
+
+
+def pbd_plan_pass(cfg: pbd_config, kind: int, prompt_lens: Sequence[int], max_new: int, grid: int,
+                  cap: int = 1 << 20):
+    """(items [n, 4] int32, cta_off [grid + 1] int32) of one pass's schedule, host only."""
+    L = load()
+    lens = np.ascontiguousarray(np.asarray(prompt_lens, dtype=np.int32))
+    items = np.zeros((cap, 4), np.int32)
+    off = np.zeros(grid + 1, np.int32)
+    n = np.zeros(1, np.int32)
+    s = L.pbd_plan_pass(C.byref(cfg), kind, len(lens), lens.ctypes.data, max_new, grid, items.ctypes.data,
+                        off.ctypes.data, cap, n.ctypes.data)
+    if s != PBD_OK:
+        raise PbdError(s, (L.pbd_last_error(None) or b"").decode())
+    return items[: int(n[0])].copy(), off
 
 
 def _ptr(t) -> int:
