@@ -143,7 +143,7 @@ def run_cpu_oracle(S, base, ad, prompt_len, D, rounds, max_seconds=None):
     from paper_2607_12422_gb300 import synth
     m = oracle.OracleModel(S, base, ad)
     prompt = synth.gen_prompts(S, [prompt_len])[0]
-    cache, p, _ = m.prefill(prompt, prompt_len + 4 * (rounds + 1) * (D + 1))
+    cache, p, _ = m.prefill(prompt, prompt_len + (rounds + 2) * (D + 1))
     L = prompt_len
     toks = 0
     done = 0
@@ -418,10 +418,11 @@ def main(args):
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        tps, sec, done, threads = run_cpu_oracle(S, base, ad, 64, D, 24, max_seconds=20)
+        P0 = Wl.prompt_lens[0]
+        tps, sec, done, threads = run_cpu_oracle(S, base, ad, P0, D, 96, max_seconds=15)
         cpu = {"value": tps, "unit": "tokens/s", "cores": threads, "kind": "oracle",
-               "sample": "%d speculative rounds (draft+verify+accept) of the same model after an untimed "
-                         "64-token prefill, %.1f s" % (done, sec)}
+               "sample": "%d speculative rounds (draft+verify+accept) of the same model after an untimed prefill "
+                         "of the workload's %d-token prompt, %.1f s (at most 96 rounds or 15 s)" % (done, P0, sec)}
 
     if rank == 0:
         line = {
