@@ -162,6 +162,19 @@ def run_cpu_oracle(S, base, ad, prompt_len, D, rounds, max_seconds=None):
     return toks / dt, dt, done, int(oracle.model.lib().orc_num_threads())
 
 
+def job_totals(dist, seconds, units, device):
+    """(slowest rank's elapsed time, units summed over ranks) of one timed region.  The ranks run
+    independent replicas, so the job's rate is the summed units over the slowest rank's time."""
+    if dist is None:
+        return float(seconds), float(units)
+    import torch
+    t = torch.tensor([float(seconds), float(units)], dtype=torch.float64, device=device)
+    mx = t.clone()
+    dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(mx[0]), float(t[1])
+
+
 def dist_setup(args):
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -342,15 +355,10 @@ def main(args):
     with ClockSampler(local) as clk:
         acc, tokens, launches, L_mean = timed_rounds(0, args.steps, args.warmup)
     torch.cuda.synchronize()
-    ms_total = acc[3]
     if dist:
-        t = torch.tensor([ms_total, float(tokens)], dtype=torch.float64, device=dev)
-        mx = t.clone()
-        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
-        dist.all_reduce(t, op=dist.ReduceOp.SUM)
-        ms_job, tok_job = float(mx[0]), float(t[1])
-    else:
-        ms_job, tok_job = ms_total, float(tokens)
+        dist.barrier()
+    ms_total = acc[3]
+    ms_job, tok_job = job_totals(dist, ms_total, tokens, dev)
     value = tok_job / (ms_job / 1e3)
     ms_per_step = ms_total / args.steps
     draft_us = 1e3 * acc[0] / args.steps
@@ -378,17 +386,21 @@ def main(args):
     traffic = traffic_for(os.path.join(ROOT, "paper_2607_12422_gb300", "csrc", "pass_kernel.cu"))
 
     # ---- end to end through the public call with host buffers
-    # (host prompt ids in, host token ids out; the binding copies the prompt to the device)
+    # (host prompt ids in, host token ids out; the binding copies the prompt to the device),
+    # whole-job over the replicas like the device-timed value
     e2e_vals = []
     for it in range(3):
+        if dist:
+            dist.barrier()
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         out, st = eng.pbd_generate([prompt], G, mode=0)
         host_tokens = out.cpu().numpy()
         dt = time.perf_counter() - t0
         assert host_tokens.shape == (1, G)
+        dt_job, tok_job_e2e = job_totals(dist, dt, G, dev)
         if it > 0:
-            e2e_vals.append(G / dt)
+            e2e_vals.append(tok_job_e2e / dt_job)
     e2e = float(np.median(e2e_vals))
 
     # ---- draft variants (Sections 4.4, 5.3 and 6): same workload, natural acceptance, one
