@@ -606,7 +606,7 @@ pbd_status pbd_plan_pass(const pbd_config *cfg, int32_t kind, int32_t batch, con
         if (h_prompt_lens[b] < 1 || h_prompt_lens[b] + max_new > cfg->max_seq_len)
             return fail(nullptr, PBD_ERR_CAPACITY, "prompt %d of %d tokens + %d exceeds max_seq_len", b,
                         h_prompt_lens[b], max_new);
-    pbd_ctx tmp;
+    pbd_ctx tmp{};  // value-initialised, as pbd_create does
     tmp.cfg = *cfg;
     tmp.dm = Dims{cfg->n_layers, cfg->hidden,      cfg->n_q_heads, cfg->n_kv_heads, cfg->head_dim,
                   cfg->intermediate, cfg->vocab, cfg->lora_rank, cfg->rms_eps,     cfg->lora_scale};
