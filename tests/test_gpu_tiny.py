@@ -240,3 +240,27 @@ def test_stalled_pass_is_reported_and_context_survives(env):
     assert int(L[0]) == P and int(n_out[0]) == 1
     out, st = eng.pbd_generate([prompt], 32, mode=0)
     assert [int(t) for t in out[0].cpu()] == oracle.greedy_generate(m, prompt, 32)
+
+
+@pytest.mark.parametrize("P,G", [(1, 1), (1, 5), (1, 17), (1, 40), (64, 3), (236, 20)],
+                         ids=["p1-g1", "p1-g5", "p1-g17", "p1-g40", "p64-g3", "p236-g20-full"])
+def test_edge_lengths(env, P, G):
+    """One-token prompts, budgets below one block (no full round), exactly one block, and a
+    prompt plus budget that fills max_seq_len (256): the speculative output is the GPU's own
+    greedy output bit for bit, and that is the oracle's greedy output up to reported near-ties."""
+    eng, m, torch = env["eng"], env["model"], env["torch"]
+    prompt = synth.gen_prompts(env["S"], [P], seed=11)[0]
+    spec, st = eng.pbd_generate([prompt], G, mode=0)
+    ar, _ = eng.pbd_generate([prompt], G, mode=1)
+    assert spec.shape[1] >= G and torch.equal(spec[0, :G], ar[0, :G])
+    assert st.emitted == G
+    ref = oracle.greedy_generate(m, prompt, G)
+    got = [int(t) for t in ar[0, :G].cpu()]
+    if got != ref:  # the first disagreement must be a near-tie of the oracle's own logits
+        j = next(i for i in range(G) if got[i] != ref[i])
+        cache, _, lg0 = m.prefill(prompt, P + G + 1, want_logits=True)
+        if j == 0:
+            lg = lg0[None]
+        else:  # the logits after ref[:j]: read-out row j - 1 of a pass over those tokens
+            _, lg, _ = m.forward(cache, P, ref[:j], False, oracle.MASK_CAUSAL, j - 1, 1, want_logits=True)
+        _check_ids([got[j]], lg, TOL)
