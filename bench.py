@@ -47,6 +47,25 @@ def peaks():
         return 6800.0, "fallback"
 
 
+def bf16_peak():
+    """Sustained dense bf16 TFLOP/s (for steps timed inside a long loop) and where it came from."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops_sustained"]), "measured (sustained)"
+    except Exception:
+        return 1700.0, "fallback (sustained)"
+
+
+def verify_flops(S, L_sum, B, D):
+    """Algorithmic FLOPs of one verify step over B sequences of D + 1 rows: every linear and the
+    tied lm_head on every row (2 per multiply-add), and causal attention (QK^T and PV, 4 d per
+    visible key and query head), row j of sequence b seeing L_b + j + 1 keys; L_sum = sum of L_b."""
+    M = B * (D + 1)
+    lin = S.n_layers * sum(i * o for i, o in (S.linear_dims(n) for n in ("q", "k", "v", "o", "gate", "up", "down")))
+    keys = (D + 1) * L_sum + B * (D + 1) * (D + 2) // 2
+    return 2 * M * (lin + S.vocab * S.hidden) + 4 * S.head_dim * S.n_q_heads * S.n_layers * keys
+
+
 def pass_bytes(S, L_mean, rows, adapter):
     """Algorithmic bytes of one pass: every weight once, the KV cache read once, the block's KV written."""
     lin = sum(S.linear_dims(n)[0] * S.linear_dims(n)[1] for n in ("q", "k", "v", "o", "gate", "up", "down"))
@@ -293,9 +312,11 @@ def measure_configs(pbd, synth, base, ad, dev, hbm, warmup):
         B = len(prompts)
         # one verify pass of the batch: every weight once, each sequence's KV once, B (D+1) rows written
         fl_v = pass_bytes(S, L_sum, B * (D + 1), False) / (hbm * 1e9) * 1e6
+        tf, _ = bf16_peak()
         out[name] = {"batch": B, "draft_us": d_us, "verify_us": v_us, "tokens_per_s": tok / (acc[3] / 1e3),
                      "mean_tokens_per_round_per_seq": tok / steps / B, "kv_tokens_mean": L_sum,
-                     "verify_roofline_frac": fl_v / v_us, "steps": steps}
+                     "verify_roofline_frac": fl_v / v_us,
+                     "verify_tensor_frac": verify_flops(S, L_sum, B, D) / (v_us * 1e-6) / (tf * 1e12), "steps": steps}
     W = synth.WORKLOADS["qwen3-0.6b-b1-p1024-dsweep-forced"]
     S = W.shape
     prompt = synth.gen_prompts(S, list(W.prompt_lens))
@@ -449,6 +470,8 @@ def main(args):
                        "draft_floor_us": floor_d, "verify_floor_us": floor_v,
                        "draft_roofline_frac": floor_d / draft_us, "verify_roofline_frac": floor_v / verify_us,
                        "draft_bytes": b_draft, "verify_bytes": b_verify, "L_mean": L_mean,
+                       "verify_tensor_frac": verify_flops(S, L_mean, 1, D) / (verify_us * 1e-6) / (bf16_peak()[0] * 1e12),
+                       "tensor_peak": "%.1f TFLOP/s bf16, %s" % bf16_peak(),
                        "mean_tokens_per_round": mean_A, "draft_over_verify": draft_us / verify_us},
             "ar": {"us_per_step": ar_us, "pass_us": ar_pass_us, "tokens_per_s": tok_ar / (acc_ar[3] / 1e3),
                    "break_even_accept": (draft_us + verify_us) / ar_us},

@@ -47,3 +47,20 @@ def test_source_hash_ignores_comments(bench, tmp_path):
     c.write_text("int f(int x) {\n  return x + 2;\n}\n")
     assert bench.source_hash(str(a)) == bench.source_hash(str(b))
     assert bench.source_hash(str(a)) != bench.source_hash(str(c))
+
+
+def test_verify_flops_closed_form(bench):
+    """2 FLOPs per multiply-add over every linear and the tied head (the pinned base parameters
+    less the 65,536 norm gains) for each of the 17 rows, plus causal attention: QK^T and PV of
+    d = 128 per visible key, 16 query heads, 28 layers, row j seeing L + j + 1 keys."""
+    S = synth.QWEN3_0_6B
+    matmul_params = oracle.base_param_count(S) - (S.n_layers * (2 * S.hidden + 2 * S.head_dim) + S.hidden)
+    assert matmul_params == 595_984_384
+    for L in (0, 512, 4096):
+        keys = sum(L + j + 1 for j in range(17))
+        assert bench.verify_flops(S, L, 1, 16) == 2 * 17 * matmul_params + 4 * 128 * 16 * 28 * keys
+    assert bench.verify_flops(S, 512, 1, 16) == 22_295_052_288
+    # a batch: the linears scale with the rows, the attention with each sequence's own keys
+    Ls = [420, 1757, 900]
+    keys = sum(L + j + 1 for L in Ls for j in range(17))
+    assert bench.verify_flops(S, sum(Ls), 3, 16) == 2 * 51 * matmul_params + 4 * 128 * 16 * 28 * keys
