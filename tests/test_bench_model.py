@@ -10,6 +10,7 @@
 import importlib.util
 import os
 
+import numpy as np
 import pytest
 
 import oracle
@@ -64,3 +65,68 @@ def test_verify_flops_closed_form(bench):
     Ls = [420, 1757, 900]
     keys = sum(L + j + 1 for L in Ls for j in range(17))
     assert bench.verify_flops(S, sum(Ls), 3, 16) == 2 * 51 * matmul_params + 4 * 128 * 16 * 28 * keys
+
+
+class _FakeEngine:
+    """Stands in for the engine in the benchmark's bookkeeping: every speculative round emits the
+    forced n + 1 tokens per sequence (2 without forcing) and reports 1, 2 and 0.01 ms for draft,
+    verify and commit (3.01 ms in all); a plain-decoding step emits one token in 2.01 ms (no
+    draft)."""
+
+    def __init__(self, shape, base, adapter, block_D, max_batch, max_seq_len, device=None, **kw):
+        self.D = block_D
+
+    def pbd_prefill(self, prompts, max_new):
+        self.G = max_new
+        self.L = np.array([len(p) for p in prompts], np.int64)
+        self.n = np.ones(len(prompts), np.int64)
+
+    def pbd_get_state(self):
+        return self.L.copy(), np.zeros_like(self.L), self.n.copy()
+
+    def pbd_bench_rounds(self, mode, warmup, steps, forced=None):
+        for i in range(steps):
+            for b in range(len(self.n)):
+                A = 1 if mode == 1 else (int(forced[i, b]) + 1 if forced is not None else 2)
+                take = min(A, self.G - self.n[b])
+                self.n[b] += take
+                self.L[b] += take
+        if mode == 1:
+            return 0.0, 2.0 * steps, 0.01 * steps, 2.01 * steps, 5
+        return 1.0 * steps, 2.0 * steps, 0.01 * steps, 3.01 * steps, 9
+
+    def close(self):
+        pass
+
+
+class _FakePbd:
+    Engine = _FakeEngine
+
+
+def test_other_workloads_bookkeeping(bench):
+    out = bench.measure_configs(_FakePbd, synth, None, None, "cpu", 6780.0, 3)
+    tf, _ = bench.bf16_peak()
+    S = synth.QWEN3_0_6B
+    for name, B, P_sum in (("qwen3-0.6b-b1-d16-p4096-g512", 1, 4096),
+                           ("qwen3-0.6b-b8-d16-p256to2048-g256", 8,
+                            sum(synth.WORKLOADS["qwen3-0.6b-b8-d16-p256to2048-g256"].prompt_lens))):
+        r = out[name]
+        W = synth.WORKLOADS[name]
+        assert r["batch"] == B and r["draft_us"] == pytest.approx(1000.0) and r["verify_us"] == pytest.approx(2000.0)
+        assert r["mean_tokens_per_round_per_seq"] == pytest.approx(2.0)  # no timed round is cut by the budget
+        assert r["tokens_per_s"] == pytest.approx(2.0 * B / 3.01e-3)
+        assert P_sum < r["kv_tokens_mean"] < P_sum + B * W.max_new
+        L = r["kv_tokens_mean"]
+        assert r["verify_roofline_frac"] == pytest.approx(bench.pass_bytes(S, L, B * 17, False) / 6780e9 / 2e-3)
+        assert r["verify_tensor_frac"] == pytest.approx(bench.verify_flops(S, L, B, 16) / 2e-3 / (tf * 1e12))
+    sweep = out["qwen3-0.6b-b1-p1024-dsweep-forced"]
+    for D in (4, 8, 16, 32):
+        row = sweep["D=%d" % D]
+        assert row["ar_us_per_token"] == pytest.approx(2010.0)
+        assert row["break_even_accept"] == pytest.approx(3000.0 / 2010.0)  # draft + verify over one step
+        assert row["mean_A_1"]["tokens_per_round"] == pytest.approx(1.0)
+        for m in ("mean_A_1", "mean_A_3", "mean_A_6"):
+            a = row[m]
+            assert a["step_us"] == pytest.approx(3010.0)
+            assert a["speedup_vs_ar"] == pytest.approx(a["tokens_per_round"] * 2010.0 / 3010.0)
+            assert a["tokens_per_s"] == pytest.approx(a["tokens_per_round"] / 3.01e-3)
