@@ -587,7 +587,7 @@ extern "C" {
 size_t pbd_workspace_bytes(const pbd_config *cfg) {
     std::string why;
     if (!valid_config(cfg, &why)) return 0;
-    pbd_ctx tmp;
+    pbd_ctx tmp{};
     tmp.cfg = *cfg;
     tmp.dm = Dims{cfg->n_layers, cfg->hidden,      cfg->n_q_heads, cfg->n_kv_heads, cfg->head_dim,
                   cfg->intermediate, cfg->vocab, cfg->lora_rank, cfg->rms_eps,     cfg->lora_scale};
