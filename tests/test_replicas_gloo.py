@@ -61,3 +61,23 @@ def test_reference_arm_other_ranks_do_no_work(monkeypatch):
     monkeypatch.setenv("WORLD_SIZE", "2")
     monkeypatch.setenv("LOCAL_RANK", "1")
     assert b.main_reference(None) == 0
+
+
+def test_reference_arm_line(monkeypatch, capsys):
+    """The reference arm (the CPU oracle on the same workload) prints one JSON line with the
+    keys the driver reads; one timed round after the 512-token prefill keeps this short."""
+    import json
+    import types
+    b = _bench()
+    for k in ("RANK", "WORLD_SIZE", "LOCAL_RANK"):
+        monkeypatch.delenv(k, raising=False)
+    args = types.SimpleNamespace(gpus=1, steps=1, warmup=0, impl="reference")
+    assert b.main_reference(args) == 0
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["metric"] == b.METRIC and line["unit"] == "tokens/s"
+    assert line["value"] > 0 and line["higher_is_better"] is True and line["steps"] == 1
+    assert line["config"]["workload"] == b.WORKLOAD and line["config"]["prompt_len"] == 512
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["value"] == line["value"]
+    assert line["cpu_baseline"]["cores"] >= 1
+    assert line["e2e"] == {"value": line["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
