@@ -219,6 +219,99 @@ def test_attention_single_visible_key_returns_its_value(attn_model):
         assert np.array_equal(out[0, h * d:(h + 1) * d], V[0, g * d:(g + 1) * d])
 
 
+class _AttnShape:
+    """The fields the oracle's config and cache need, for attention-only pins at any (d, Hq, Hkv)."""
+
+    def __init__(self, d, hq, hkv):
+        self.n_layers, self.hidden, self.n_q_heads, self.n_kv_heads, self.head_dim = 1, hq * d, hq, hkv, d
+        self.intermediate, self.vocab, self.rms_eps, self.rope_theta = 4 * d, 16, 1e-6, 1e6
+        self.lora_rank, self.lora_alpha = 8, 16.0
+
+
+class _AttnHolder:
+    def __init__(self, shape):
+        self.shape, self.cfg = shape, om.make_config(shape)
+
+
+def _visible(mode, L, n, i):
+    """Key positions row i of an n-row block at L may read, written out from the masks' definitions
+    (Section 3 and Appendix A.4): causal rows see every earlier position and themselves; under the
+    draft mask the pending row (i = 0) sees the cache and itself, a mask row the whole block."""
+    if mode == oracle.MASK_CAUSAL or i == 0:
+        return list(range(L + i + 1))
+    return list(range(L + n))
+
+
+@pytest.mark.parametrize("d,hq,hkv", [(64, 4, 2), (128, 16, 8), (32, 3, 1), (64, 6, 3)])
+@pytest.mark.parametrize("offset", [0.0, 100.0])
+def test_attention_weights_follow_exp_of_scaled_scores(d, hq, hkv, offset):
+    """Scores built as s_k = offset + ln(w_k) with integer w_k make the softmax weights exactly
+    w_k / sum(w) over the visible keys, so every output is a known mixture of the values.
+
+    Query head h is c * e_{j(h)} and key k of KV group g is sum_j a_{k,j} e_j with
+    a_{k,j} = sqrt(d) (offset + ln w[g][k][j]) / c: the score q.k / sqrt(d) is offset + ln w.
+    A scale of 1/d or none, a wrong exponent base, a wrong query-head to KV-group map or a
+    masked key taken in changes the mixture; at offset 100 the scores overflow exp in fp32
+    unless the row maximum is subtracted first (exp(100) > 3.4e38), so a softmax without the
+    max shift returns NaN.  Values are bf16 numbers; the output is rounded once to bf16."""
+    S = _AttnShape(d, hq, hkv)
+    holder = _AttnHolder(S)
+    grp = hq // hkv
+    L, D = 5, 3
+    n = D + 1
+    T = L + n
+    rng = np.random.default_rng(100 + d + hq)
+    # weights 1..9 per (group, key, query column j); query head h uses column j(h) = h % grp
+    w = rng.integers(1, 10, size=(hkv, T, grp)).astype(np.float64)
+    c = 4.0
+    K = np.zeros((T, hkv * d), np.float64)
+    for g in range(hkv):
+        for k in range(T):
+            for j in range(grp):
+                K[k, g * d + j] = math.sqrt(d) * (offset + math.log(w[g, k, j])) / c
+    V = _bf16_round(rng.standard_normal((T, hkv * d)))
+    cache = om.OracleCache(holder, T)
+    cache.write(0, 0, K.astype(np.float32), V)
+    q = np.zeros((n, hq * d), np.float32)
+    for h in range(hq):
+        q[:, h * d + h % grp] = c
+    for mode in (oracle.MASK_CAUSAL, oracle.MASK_BLOCK_DRAFT):
+        out = _attention(S, cache, L, n, mode, q)
+        assert np.all(np.isfinite(out)), (mode, offset)
+        for i in range(n):
+            vis = _visible(mode, L, n, i)
+            for h in range(hq):
+                g = h // grp
+                wk = w[g, vis, h % grp]
+                ref = (wk[:, None] * V[vis, g * d:(g + 1) * d].astype(np.float64)).sum(0) / wk.sum()
+                got = out[i, h * d:(h + 1) * d].astype(np.float64)
+                # bf16 rounding of the output (2^-9 relative) plus the fp32 scores' relative error
+                # (~1e-7 of |s| <= 103) carried through exp
+                assert np.allclose(got, ref, rtol=2 ** -8, atol=2 ** -8 * np.abs(ref).max() + 1e-6), (mode, i, h)
+
+
+def test_attention_two_keys_three_to_one():
+    """Two visible keys, scores 0 and ln 3: weights 1/4 and 3/4, output v0/4 + 3 v1/4 (the row at
+    position 1 of a prompt, causal).  A 1/d scale would give weights 0.466 / 0.534 at d = 64."""
+    S = _AttnShape(64, 2, 1)
+    holder = _AttnHolder(S)
+    cache = om.OracleCache(holder, 4)
+    d = 64
+    K = np.zeros((2, d), np.float32)
+    K[1, 0] = math.sqrt(d) * math.log(3.0) / 2.0
+    V = np.zeros((2, d), np.float32)
+    V[0, :] = 1.0
+    V[1, :] = 2.0
+    cache.write(0, 0, K, V)
+    q = np.zeros((2, 2 * d), np.float32)
+    q[:, 0] = 2.0
+    q[:, d] = 2.0
+    out = _attention(S, cache, 0, 2, oracle.MASK_CAUSAL, q)
+    # row 1 mixes 1.0 and 2.0 with weights 1/4, 3/4 = 1.75 exactly (a bf16 number)
+    assert np.allclose(out[1], 1.75, rtol=0, atol=2 ** -7)
+    assert np.all(out[0] == 1.0)
+
+
 # ---------------------------------------------------------------- SwiGLU
 
 def _swiglu(g, u):
