@@ -25,7 +25,10 @@ size_t pbd_op_linear_workspace_bytes(int32_t M, int32_t K, int32_t N, int32_t r)
  * d_a == NULL or d_b == NULL (or r == 0) switches the delta off.  Runs the same tensor-core
  * kernel as the decoder passes (K split in 256-wide slices, fp32 partial sums in the workspace,
  * fixed-order reduction).  Requirements: N % 128 == 0, K % 64 == 0, 1 <= M <= 4096, r <= 32.
- * The workspace (d_ws, >= pbd_op_linear_workspace_bytes, 1024-byte aligned) is scratch. */
+ * The workspace (d_ws, >= pbd_op_linear_workspace_bytes, 1024-byte aligned) is scratch; its first
+ * word is the kernel's status word, cleared by each call and read by pbd_op_status.
+ * The return value covers argument checks and launches only: a bounded device wait that ran out
+ * is reported by pbd_op_status(d_ws, ...) after the call (before the next call on d_ws). */
 pbd_status pbd_op_linear(int32_t M, int32_t K, int32_t N, int32_t r, float scale, const void *d_x, const void *d_w,
                          const void *d_a, const void *d_b, void *d_y, void *d_ws, size_t ws_bytes, void *d_stream);
 
@@ -56,9 +59,14 @@ pbd_status pbd_op_linear(int32_t M, int32_t K, int32_t N, int32_t r, float scale
  * Within 16 MiB fit, for instance, an N = 6144, K = 1024 weight with r = 16 up to M = 39, and
  * an N = 1024, K = 3072 weight with r = 16 up to M = 194.
  *
- * Zeroing: every call clears, on d_stream, the parts of the scratch that must start at zero
- * (the kernel's status word and the adapter's row tile); everything else is overwritten before
- * it is read, so a call never sees an earlier call's data.
+ * Zeroing: every call clears, on d_stream, the one part of the scratch that must start at zero,
+ * the kernel's status word.  Every other byte a call reads (the re-tiled weight and adapter rows,
+ * the partial sums) is written by that same call first, so a call never sees an earlier call's
+ * data.
+ *
+ * Device errors: as for pbd_op_linear, the return value covers argument checks and launches;
+ * pbd_op_linear_static_status reports a device wait that ran out.  Ask before the next call on
+ * the device, which clears the status word.
  *
  * Concurrency: all calls on one device share the same scratch.  Two calls whose work can
  * overlap in time on the device (different streams without an ordering between them, or
@@ -72,15 +80,33 @@ pbd_status pbd_op_linear(int32_t M, int32_t K, int32_t N, int32_t r, float scale
 pbd_status pbd_op_linear_static(int32_t M, int32_t K, int32_t N, int32_t r, float scale, const void *d_x,
                                 const void *d_w, const void *d_a, const void *d_b, void *d_y, void *d_stream);
 
+/* Device status of the last pbd_op_linear_static call on the current device: waits for d_stream,
+ * then reads the status word in the library's static scratch.  PBD_OK (and *h_device_code = 0)
+ * when no kernel latched an error; PBD_ERR_DEVICE with the latched code (the DEV_* values of the
+ * pass kernel: 1 copy, 2 accumulation, 3 ring slot, 6 inputs) in *h_device_code otherwise, in
+ * which case that call's y is invalid; PBD_ERR_STATE if no call was made on this device yet;
+ * PBD_ERR_CUDA if the stream failed.  h_device_code may be NULL.  Allocates nothing. */
+pbd_status pbd_op_linear_static_status(void *d_stream, int32_t *h_device_code);
+
 /* Workspace bytes pbd_op_lm_head_argmax needs (0 if unsupported). */
 size_t pbd_op_lm_head_workspace_bytes(int32_t M, int32_t H, int32_t V);
 
 /* Tied lm_head with greedy readout (Section 3, step 4 uses the verifier's top-1 token):
  *     logits = x E^T (fp32, never rounded),  ids[m] = argmax_v logits[m, v], lowest v on ties.
  * d_x [M, H] and d_embed [V, H] bf16 row-major; d_ids [M] int32; d_logits_opt [M, V] fp32 or
- * NULL.  Requirements: V % 128 == 0, H % 64 == 0, 1 <= M <= 256. */
+ * NULL.  Requirements: V % 128 == 0, H % 64 == 0, 1 <= M <= 256.  The workspace's first word is
+ * the kernel's status word: pbd_op_status(d_ws, ...) reports a device wait that ran out. */
 pbd_status pbd_op_lm_head_argmax(int32_t M, int32_t H, int32_t V, const void *d_x, const void *d_embed,
                                  int32_t *d_ids, float *d_logits_opt, void *d_ws, size_t ws_bytes, void *d_stream);
+
+/* Device status of the last pbd_op_linear or pbd_op_lm_head_argmax call that used the
+ * workspace d_ws (the 1024-byte-aligned pointer that call was given): waits for d_stream, then
+ * reads the status word at the start of d_ws.  PBD_OK when no kernel latched an error;
+ * PBD_ERR_DEVICE with the latched code in *h_device_code (may be NULL) otherwise, and that call's
+ * outputs are invalid; PBD_ERR_INVALID_ARG for a null or misaligned d_ws; PBD_ERR_CUDA if the
+ * stream failed.  A device wait bounded at one second that runs out is the only way these kernels
+ * latch an error (the kernels' bounds on their inputs are checked on the host). */
+pbd_status pbd_op_status(const void *d_ws, void *d_stream, int32_t *h_device_code);
 
 /* Message of the last failed pbd_op_* call on this thread ("" if none). */
 const char *pbd_op_last_error(void);

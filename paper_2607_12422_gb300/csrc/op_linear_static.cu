@@ -125,17 +125,13 @@ extern "C" pbd_status pbd_op_linear_static(int32_t M, int32_t K, int32_t N, int3
     P.k_splits = p.k_splits;
     P.rows_alloc = M;
     P.n_total = N + rr;
-    const size_t tile_row_bytes = (size_t)(K / KT) * TILE_BYTES;
     uint8_t *tiles = ws + p.tiles_off;
 
     cudaError_t e;
-    // What must start at zero on every call: the status word, which the kernel only ever raises,
-    // and the adapter's row tile, whose rows past r would otherwise hold an earlier call's data.
-    // The main tiles and the partial sums are overwritten in full before they are read.
+    // What must start at zero on every call: the status word, which the kernel only ever raises.
+    // The weight tiles and the partial sums this call reads are written by this call first (the
+    // kernel copies only the adapter tile's first r rows, and stores only rows it computed).
     if ((e = cudaMemsetAsync(status, 0, 256, st)) != cudaSuccess) return fail_cuda("clear status", e);
-    if (lora && (e = cudaMemsetAsync(tiles + (size_t)(N / TILE_ROWS) * tile_row_bytes, 0, tile_row_bytes, st)) !=
-                    cudaSuccess)
-        return fail_cuda("clear adapter tile", e);
     if ((e = launch_repack_tiled(d_w, N, K, tiles, 0, st)) != cudaSuccess) return fail_cuda("repack W", e);
     if (lora && (e = launch_repack_tiled(d_a, rr, K, tiles, N, st)) != cudaSuccess) return fail_cuda("repack A", e);
     if ((e = launch_linear_partials(&map, bn, w, lora ? 1 : 0, M, P, status, st)) != cudaSuccess)
@@ -143,4 +139,24 @@ extern "C" pbd_status pbd_op_linear_static(int32_t M, int32_t K, int32_t N, int3
     if ((e = launch_linear_finalize(P, M, N, rr, scale, d_b, d_y, st)) != cudaSuccess)
         return fail_cuda("finalize", e);
     return PBD_OK;
+}
+
+extern "C" pbd_status pbd_op_linear_static_status(void *d_stream, int32_t *h_device_code) {
+    if (h_device_code) *h_device_code = 0;
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return fail_cuda("cudaGetDevice", e);
+    uint8_t *ws = nullptr;
+    {
+        std::lock_guard<std::mutex> lock(g_setup_mu);
+        if (dev >= 0 && dev < MAX_DEVICES) ws = g_scratch[dev];
+    }
+    if (ws == nullptr)
+        return fail(PBD_ERR_STATE, "pbd_op_linear_static_status: no pbd_op_linear_static call on this device yet");
+    int code = 0;
+    const pbd_status s = read_device_code(reinterpret_cast<const int *>(ws), static_cast<cudaStream_t>(d_stream), &code,
+                                          "pbd_op_linear_static_status");
+    if (s != PBD_OK) return s;
+    if (h_device_code) *h_device_code = code;
+    return code == 0 ? PBD_OK : device_fail(code, "pbd_op_linear_static");
 }

@@ -83,6 +83,42 @@ bool plan_linear(int M, int K, int N, int r, LinearPlan *p) {
 
 }  // namespace
 
+namespace pbd {
+
+// Waits for d_stream, then reads the status word a kernel may have latched (a DEV_* code).
+pbd_status read_device_code(const int *d_status, cudaStream_t st, int *code, const char *who) {
+    cudaError_t e = cudaStreamSynchronize(st);
+    if (e == cudaSuccess) e = cudaMemcpy(code, d_status, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) {
+        char b[128];
+        snprintf(b, sizeof b, "%s: reading the status word", who);
+        return op_fail(PBD_ERR_CUDA, b, e);
+    }
+    return PBD_OK;
+}
+
+const char *device_code_name(int code) {
+    switch (code) {
+        case DEV_TIMEOUT_LOAD: return "a weight or operand copy never completed";
+        case DEV_TIMEOUT_MMA: return "a tensor-core accumulation never completed";
+        case DEV_TIMEOUT_SLOT: return "a shared-memory ring slot was never released";
+        case DEV_BAD_TOKEN: return "token id outside the vocabulary";
+        case DEV_BAD_POSITION: return "position beyond the reserved KV pages";
+        case DEV_TIMEOUT_DEP: return "a work item's inputs never completed";
+        default: return "unknown device code";
+    }
+}
+
+pbd_status device_fail(int code, const char *who) {
+    char b[256];
+    snprintf(b, sizeof b, "%s: device status %d latched by a kernel (%s); the outputs of that call are invalid", who,
+             code, device_code_name(code));
+    g_op_err = b;
+    return PBD_ERR_DEVICE;
+}
+
+}  // namespace pbd
+
 extern "C" {
 
 size_t pbd_op_linear_workspace_bytes(int32_t M, int32_t K, int32_t N, int32_t r) {
@@ -171,6 +207,18 @@ pbd_status pbd_op_lm_head_argmax(int32_t M, int32_t H, int32_t V, const void *d_
     if ((e = launch_argmax_reduce(tmax, targ, V / TILE_ROWS, M, d_ids, st)) != cudaSuccess)
         return op_fail(PBD_ERR_CUDA, "argmax", e);
     return PBD_OK;
+}
+
+pbd_status pbd_op_status(const void *d_ws, void *d_stream, int32_t *h_device_code) {
+    if (h_device_code) *h_device_code = 0;
+    if (!d_ws || (reinterpret_cast<uintptr_t>(d_ws) & 1023))
+        return op_fail(PBD_ERR_INVALID_ARG, "pbd_op_status: workspace missing or misaligned");
+    int code = 0;
+    pbd_status s = read_device_code(static_cast<const int *>(d_ws), static_cast<cudaStream_t>(d_stream), &code,
+                                    "pbd_op_status");
+    if (s != PBD_OK) return s;
+    if (h_device_code) *h_device_code = code;
+    return code == 0 ? PBD_OK : device_fail(code, "pbd_op_status");
 }
 
 const char *pbd_op_last_error(void) { return g_op_err.c_str(); }

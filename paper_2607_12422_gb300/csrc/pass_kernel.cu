@@ -318,10 +318,12 @@ __device__ __forceinline__ const bf16 *tiled_at(const bf16 *tiles, int K, int v,
 
 // ------------------------------------------------------------------ work items
 
-// token / mask-embedding row -> residual h and its per-tile sums of squares
+// token / mask-embedding row -> residual h and its per-tile sums of squares.  A mask row is
+// id -1 and exists only in adapter-on (draft) passes; any other id outside [0, V) latches
+// DEV_BAD_TOKEN and reads row 0 instead of memory outside the embedding.
 __device__ __noinline__ void do_embed(const MKParams &P, int m, int cw, int lane) {
     int tok = P.ids[m];
-    if (tok >= P.dm.V) {
+    if (tok >= P.dm.V || tok < -1 || (tok == -1 && !P.pd.adapter)) {
         latch_error(P.status, DEV_BAD_TOKEN);
         tok = 0;
     }

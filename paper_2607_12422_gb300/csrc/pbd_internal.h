@@ -8,6 +8,8 @@
 
 #include <vector>
 
+#include "../../include/pbd.h"
+
 namespace pbd {
 
 constexpr int PAGE = 16;           // KV page length in tokens
@@ -192,5 +194,10 @@ cudaError_t configure_linear_kernels();
 
 // Records the message pbd_op_last_error() returns on this thread.
 void op_record_error(const char *msg);
+
+// Single-op status words: wait for the stream and read the latched DEV_* code; turn a nonzero
+// code into PBD_ERR_DEVICE with its message (pbd_op_last_error()).
+pbd_status read_device_code(const int *d_status, cudaStream_t st, int *code, const char *who);
+pbd_status device_fail(int code, const char *who);
 
 }  // namespace pbd

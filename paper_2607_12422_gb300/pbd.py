@@ -110,6 +110,10 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     L.pbd_op_last_error.restype = C.c_char_p
     L.pbd_op_linear_static.argtypes = [I32, I32, I32, I32, C.c_float, P, P, P, P, P, P]
     L.pbd_op_linear_static.restype = C.c_int
+    L.pbd_op_status.argtypes = [P, P, P]
+    L.pbd_op_status.restype = C.c_int
+    L.pbd_op_linear_static_status.argtypes = [P, P]
+    L.pbd_op_linear_static_status.restype = C.c_int
     for name in ("pbd_create", "pbd_destroy", "pbd_prefill", "pbd_draft_block", "pbd_verify_block",
                  "pbd_accept_commit", "pbd_decode_step", "pbd_generate", "pbd_get_state", "pbd_get_tokens",
                  "pbd_read_kv", "pbd_sync", "pbd_op_linear", "pbd_op_lm_head_argmax"):
@@ -125,8 +129,14 @@ def _ws(torch, nbytes, device):
     return buf, buf.data_ptr() + off
 
 
+def _raise_if(L, s):
+    if s != PBD_OK:
+        raise PbdError(s, L.pbd_op_last_error().decode())
+
+
 def pbd_op_linear(x, W, A=None, B=None, scale: float = 2.0):
-    """y = bf16(x W^T + scale * bf16(x A^T) B^T) on the GPU (torch bf16 device tensors in, out)."""
+    """y = bf16(x W^T + scale * bf16(x A^T) B^T) on the GPU (torch bf16 device tensors in, out).
+    Waits for the result and raises PbdError(PBD_ERR_DEVICE) if a kernel latched an error."""
     import torch
     L = load()
     M, K = x.shape
@@ -135,40 +145,55 @@ def pbd_op_linear(x, W, A=None, B=None, scale: float = 2.0):
     need = L.pbd_op_linear_workspace_bytes(M, K, N, r)
     if need == 0:
         raise PbdError(1, "pbd_op_linear: unsupported sizes")
-    buf, ws = _ws(torch, need, x.device)
-    y = torch.empty(M, N, dtype=torch.bfloat16, device=x.device)
-    st = torch.cuda.current_stream(x.device).cuda_stream
-    s = L.pbd_op_linear(M, K, N, r, scale, x.data_ptr(), W.data_ptr(), _ptr(A) if r else None,
-                        _ptr(B) if r else None, y.data_ptr(), ws, need, st)
-    if s != PBD_OK:
-        raise PbdError(s, L.pbd_op_last_error().decode())
-    torch.cuda.synchronize(x.device)
+    with torch.cuda.device(x.device):  # the library runs on the current device
+        buf, ws = _ws(torch, need, x.device)
+        y = torch.empty(M, N, dtype=torch.bfloat16, device=x.device)
+        st = torch.cuda.current_stream(x.device).cuda_stream
+        _raise_if(L, L.pbd_op_linear(M, K, N, r, scale, x.data_ptr(), W.data_ptr(), _ptr(A) if r else None,
+                                     _ptr(B) if r else None, y.data_ptr(), ws, need, st))
+        _raise_if(L, L.pbd_op_status(ws, st, None))
     del buf
     return y
 
 
 def pbd_op_linear_static(x, W, A=None, B=None, scale: float = 2.0, y=None, sync: bool = True):
     """pbd_op_linear through the entry point that takes no workspace (the library's own static
-    scratch); y [M, N] bf16 is the caller's output tensor (allocated here when not given)."""
+    scratch); y [M, N] bf16 is the caller's output tensor (allocated here when not given).
+    With sync, waits and raises PbdError(PBD_ERR_DEVICE) if the kernel latched an error; without
+    it the caller asks pbd_op_linear_static_status before the next call."""
     import torch
     L = load()
     M, K = x.shape
     N = W.shape[0]
     r = A.shape[0] if (A is not None and B is not None) else 0
-    if y is None:
-        y = torch.empty(M, N, dtype=torch.bfloat16, device=x.device)
-    st = torch.cuda.current_stream(x.device).cuda_stream
-    s = L.pbd_op_linear_static(M, K, N, r, scale, x.data_ptr(), W.data_ptr(), _ptr(A) if r else None,
-                               _ptr(B) if r else None, y.data_ptr(), st)
-    if s != PBD_OK:
-        raise PbdError(s, L.pbd_op_last_error().decode())
-    if sync:
-        torch.cuda.synchronize(x.device)
+    with torch.cuda.device(x.device):  # the library picks its scratch by the current device
+        if y is None:
+            y = torch.empty(M, N, dtype=torch.bfloat16, device=x.device)
+        st = torch.cuda.current_stream(x.device).cuda_stream
+        _raise_if(L, L.pbd_op_linear_static(M, K, N, r, scale, x.data_ptr(), W.data_ptr(), _ptr(A) if r else None,
+                                            _ptr(B) if r else None, y.data_ptr(), st))
+        if sync:
+            _raise_if(L, L.pbd_op_linear_static_status(st, None))
     return y
 
 
+def pbd_op_linear_static_status(device=None) -> int:
+    """Device code of the last pbd_op_linear_static call on `device` (0 = none); raises PbdError
+    on PBD_ERR_DEVICE, PBD_ERR_STATE (no call yet) or PBD_ERR_CUDA."""
+    import torch
+    L = load()
+    dev = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
+    code = C.c_int32(0)
+    with torch.cuda.device(dev):
+        s = L.pbd_op_linear_static_status(torch.cuda.current_stream(dev).cuda_stream, C.byref(code))
+    if s != PBD_OK:
+        raise PbdError(s, L.pbd_op_last_error().decode())
+    return code.value
+
+
 def pbd_op_lm_head_argmax(x, E, want_logits: bool = False):
-    """(argmax ids [M] int32, logits [M, V] fp32 or None) of x E^T on the GPU."""
+    """(argmax ids [M] int32, logits [M, V] fp32 or None) of x E^T on the GPU.
+    Waits for the result and raises PbdError(PBD_ERR_DEVICE) if a kernel latched an error."""
     import torch
     L = load()
     M, H = x.shape
@@ -176,14 +201,14 @@ def pbd_op_lm_head_argmax(x, E, want_logits: bool = False):
     need = L.pbd_op_lm_head_workspace_bytes(M, H, V)
     if need == 0:
         raise PbdError(1, "pbd_op_lm_head_argmax: unsupported sizes")
-    buf, ws = _ws(torch, need, x.device)
-    ids = torch.empty(M, dtype=torch.int32, device=x.device)
-    lg = torch.empty(M, V, dtype=torch.float32, device=x.device) if want_logits else None
-    st = torch.cuda.current_stream(x.device).cuda_stream
-    s = L.pbd_op_lm_head_argmax(M, H, V, x.data_ptr(), E.data_ptr(), ids.data_ptr(), _ptr(lg), ws, need, st)
-    if s != PBD_OK:
-        raise PbdError(s, L.pbd_op_last_error().decode())
-    torch.cuda.synchronize(x.device)
+    with torch.cuda.device(x.device):
+        buf, ws = _ws(torch, need, x.device)
+        ids = torch.empty(M, dtype=torch.int32, device=x.device)
+        lg = torch.empty(M, V, dtype=torch.float32, device=x.device) if want_logits else None
+        st = torch.cuda.current_stream(x.device).cuda_stream
+        _raise_if(L, L.pbd_op_lm_head_argmax(M, H, V, x.data_ptr(), E.data_ptr(), ids.data_ptr(), _ptr(lg), ws,
+                                             need, st))
+        _raise_if(L, L.pbd_op_status(ws, st, None))
     del buf
     return ids, lg
 

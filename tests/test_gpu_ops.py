@@ -92,3 +92,29 @@ def test_lm_head_argmax_matches_oracle(torch_dev, M, H, V):
         srt = np.sort(ref[m])
         if srt[-1] - srt[-2] > 1e-4:
             assert ids[m] == int(np.argmax(ref[m]))
+
+
+def test_op_status_reports_a_latched_device_code(torch_dev):
+    """pbd_op_status maps the workspace's status word to PBD_ERR_DEVICE with the code (a word set
+    here by hand: no kernel is made to fail), leaves a clean word PBD_OK, and a real call's word
+    is clean."""
+    torch = torch_dev
+    from paper_2607_12422_gb300 import pbd
+    L = pbd.load()
+    buf = torch.zeros(4096, dtype=torch.uint8, device="cuda")
+    off = (-buf.data_ptr()) % 1024
+    ws = buf[off:off + 1024]
+    st = torch.cuda.current_stream().cuda_stream
+    code = C.c_int32(-1)
+    assert L.pbd_op_status(ws.data_ptr(), st, C.byref(code)) == 0 and code.value == 0
+    ws.view(torch.int32)[0] = 6  # DEV_TIMEOUT_DEP
+    assert L.pbd_op_status(ws.data_ptr(), st, C.byref(code)) == 6 and code.value == 6
+    assert b"device status 6" in L.pbd_op_last_error()
+    # a real call: its own status word starts clean and stays clean
+    rng = np.random.default_rng(3)
+    x = _to_dev(torch, _bf16(rng, (5, 256), 1.0))
+    W = _to_dev(torch, _bf16(rng, (128, 256), 0.02))
+    y = pbd.pbd_op_linear(x, W)  # raises on a latched code
+    assert y.shape == (5, 128)
+    ids, _ = pbd.pbd_op_lm_head_argmax(x, W)
+    assert ids.shape == (5,)

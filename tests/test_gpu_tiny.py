@@ -242,6 +242,31 @@ def test_stalled_pass_is_reported_and_context_survives(env):
     assert [int(t) for t in out[0].cpu()] == oracle.greedy_generate(m, prompt, 32)
 
 
+def test_out_of_range_token_ids_are_latched_and_context_survives(env):
+    """The device bounds latch on token ids (the one input the host cannot check: it is device
+    memory): a prompt holding id V, or a negative id, is embedded from row 0 instead of read out
+    of bounds, the prefill reports PBD_ERR_DEVICE with DEV_BAD_TOKEN (4), and so does a verify
+    pass given a drafted id of V.  The same context then decodes a valid prompt exactly."""
+    eng, m, prompt, pbd = env["eng"], env["model"], env["prompts"][0], env["pbd"]
+    V = env["S"].vocab
+    for bad in (V, -5, -1):  # -1 is a mask row, valid only in a draft pass
+        p = np.array(prompt, np.int32).copy()
+        p[3] = bad
+        with pytest.raises(pbd.PbdError) as ei:
+            eng.pbd_prefill([p], max_new=16)
+        assert ei.value.status == 6 and "device status 4" in str(ei.value), bad
+    eng.pbd_prefill([prompt], max_new=16)
+    d_ids, _ = eng.pbd_draft_block()
+    drafts = d_ids.clone()
+    drafts[0, 2] = V
+    eng.pbd_verify_block(drafts=drafts)
+    with pytest.raises(pbd.PbdError) as ei:
+        eng.pbd_sync()
+    assert ei.value.status == 6 and "device status 4" in str(ei.value)
+    out, st = eng.pbd_generate([prompt], 32, mode=0)
+    assert [int(t) for t in out[0].cpu()] == oracle.greedy_generate(m, prompt, 32)
+
+
 @pytest.mark.parametrize("P,G", [(1, 1), (1, 5), (1, 17), (1, 40), (64, 3), (236, 20)],
                          ids=["p1-g1", "p1-g5", "p1-g17", "p1-g40", "p64-g3", "p236-g20-full"])
 def test_edge_lengths(env, P, G):

@@ -71,6 +71,13 @@ def test_create_rejects_bad_arguments_without_gpu(lib):
     assert lib.pbd_version().startswith(b"pbd sm_103a")
 
 
+def test_op_status_validates_arguments_without_gpu(lib):
+    code = C.c_int32(-1)
+    assert lib.pbd_op_status(None, None, C.byref(code)) == 1 and code.value == 0
+    assert lib.pbd_op_status(0x100010, None, None) == 1  # not 1024-byte aligned
+    assert b"pbd_op_status" in lib.pbd_op_last_error()
+
+
 def test_state_calls_need_a_context(lib):
     assert lib.pbd_draft_block(None, None, None) == 1
     assert lib.pbd_sync(None) == 1

@@ -60,8 +60,9 @@ def test_static_scratch_matches_workspace_linear_on_consecutive_calls(lib):
     torch = pytest.importorskip("torch")
     if not torch.cuda.is_available():
         pytest.skip("no GPU")
-    # call 1 fills most of the scratch (gate|up-shaped, rank 16); call 2 is smaller with rank 8,
-    # so its adapter tile would hold call 1's rows 8..15 if they were not cleared
+    # call 1 fills most of the scratch (gate|up-shaped, rank 16); call 2 has another shape (fewer
+    # rows, a longer K in more slices, rank 8), so its tiles and partial sums lie on bytes call 1
+    # wrote: its result must not depend on them
     cases = [(17, 1024, 6144, 16, 11), (5, 3072, 1024, 8, 12)]
     inputs = []
     for M, K, N, r, seed in cases:
@@ -79,6 +80,7 @@ def test_static_scratch_matches_workspace_linear_on_consecutive_calls(lib):
         pbd.pbd_op_linear_static(x, W, A, B, 2.0, y=y, sync=False)
     torch.cuda.synchronize()
     assert torch.cuda.memory_allocated() == before  # the calls took no memory from torch
+    assert pbd.pbd_op_linear_static_status() == 0  # no kernel latched a device error
     for (x, W, A, B, y), (M, K, N, r, _) in zip(inputs, cases):
         ref = pbd.pbd_op_linear(x, W, A, B, 2.0).float().cpu().numpy()
         got = y.float().cpu().numpy()
