@@ -189,12 +189,14 @@ pbd_status pbd_time_pass(pbd_ctx *ctx, int32_t kind, int32_t iters, double *h_ms
 
 /* Timeline of one pass of the persistent kernel (a profiling aid; the paper's Appendix A.5 profiles
  * draft and verify forward latency).  On a prefilled context, runs one draft (kind 0), verify (1)
- * or plain-decoding (2) pass without advancing the state, recording for every work item eight
+ * or plain-decoding (2) pass without advancing the state, recording for every work item sixteen
  * %globaltimer stamps in ns: start, inputs complete, main work done, end, then per item kind
- * (linear: operand staged, accumulator ready, completion counted, reduction done; attention:
- * K/V landed, V converted, completion counted, merge done; 0 when not reached).  h_items
- * receives per item {op | lin << 8 | layer << 16, a, b, c}, h_trace the stamps [n, 8], both in
- * the schedule's order; at most `cap` items; *h_n the item count. */
+ * (linear: operand staged, accumulator ready, partials stored, reduction done, norm scales or
+ * act words ready, first reduced row's partial sums present, its outputs computed, reduction's
+ * stores issued; attention: K/V landed, V converted, all splits stored, merge done, block pages
+ * requested, q fragments loaded, softmax done, partials stored, merge inputs loaded; 0 when not
+ * reached).  h_items receives per item {op | lin << 8 | layer << 16, a, b, c}, h_trace the
+ * stamps [n, 16], both in the schedule's order; at most `cap` items; *h_n the item count. */
 pbd_status pbd_trace_pass(pbd_ctx *ctx, int32_t kind, int32_t *h_items, uint64_t *h_trace, int32_t cap,
                           int32_t *h_n);
 

@@ -123,13 +123,18 @@ struct MKParams {
     int att_splits_alloc;
     float att_scale;           // 1/sqrt(head_dim)
     int *status, *abort;
-    unsigned long long *trace;  // optional: 4 timestamps per item (start, inputs ready, work done, end)
+    unsigned long long *trace;  // optional: MK_STAMPS timestamps per item (see pbd_internal.h)
     // launch geometry
     int bn, nslot, ring_bytes, union_bytes;
     uint32_t tmem_cols;
 };
 
 __device__ __forceinline__ bool aborted(const MKParams &P) { return ld_relaxed(P.abort) != 0; }
+
+// sub-step timestamp of a traced pass (st = the item's stamp row, null when not tracing)
+__device__ __forceinline__ void stamp_at(unsigned long long *st, int k) {
+    if (st) st[k] = globaltimer_ns();
+}
 
 __device__ __forceinline__ void raise_abort(const MKParams &P, int code) {
     latch_error(P.status, code);
@@ -346,7 +351,7 @@ __device__ __noinline__ void do_embed(const MKParams &P, int m, int cw, int lane
 // 64j..64j+63 of the slice) holds row m at m*128 bytes, 16-byte chunk c at (c ^ (m & 7)) * 16.
 // Row m of the q|k|v and gate|up inputs is RMSNorm(h_m) * gain, computed here on the fly.
 __device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int slice, uint8_t *sb, float *s_rms, int ct,
-                                     int a0, int na, bool need_rms) {
+                                     int a0, int na, bool need_rms, unsigned long long *st) {
     constexpr int U = 4;  // chunks in flight per thread
     const int M = P.pd.M;
     const int k0 = (slice * P.katoms[lin] + a0) * KT;
@@ -373,6 +378,7 @@ __device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int 
     if (norm && need_rms) {
         for (int m = ct; m < M; m += CT) s_rms[m] = row_rms(P, m);
         bar_compute();
+        if (ct == 0) stamp_at(st, 8);
     }
     for (int q0 = ct; q0 < chunks; q0 += U * CT) {
         if (q0 != ct) issue(q0);
@@ -399,7 +405,8 @@ __device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int 
 // The down projection's activation tile from the tagged act words of this layer's gate|up
 // reductions (same layout as build_b): every 16-byte chunk of 8 features is four words, read
 // again until all carry the tag (bounded).  No completion counter precedes it.
-__device__ __noinline__ void build_b_act(const MKParams &P, int slice, uint8_t *sb, int ct, uint32_t tag) {
+__device__ __noinline__ void build_b_act(const MKParams &P, int slice, uint8_t *sb, int ct, uint32_t tag,
+                                         unsigned long long *st) {
     constexpr int U = 4;  // chunks in flight per thread
     const int M = P.pd.M, ld = P.dm.I;
     const int k0 = slice * P.katoms[3] * KT;
@@ -446,6 +453,7 @@ __device__ __noinline__ void build_b_act(const MKParams &P, int slice, uint8_t *
                 break;
             }
         }
+        if (q0 == ct && ct == 0) stamp_at(st, 8);
 #pragma unroll
         for (int u = 0; u < U; ++u) {
             const int q = q0 + u * CT;
@@ -461,7 +469,7 @@ __device__ __noinline__ void build_b_act(const MKParams &P, int slice, uint8_t *
 // q|k|v tile: adapter delta, bf16, per-head RMSNorm + RoPE for q and k, store q / paged K, V
 template <int DH, bool AD>
 __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, int cw, int lane, int m0, int mstep,
-                                       uint32_t tag) {
+                                       uint32_t tag, unsigned long long *st) {
     constexpr int E = DH / 32;
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r;
@@ -487,6 +495,8 @@ __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, 
             for (int j = 0; j < E; ++j) br[j] = load_brow(lb + (size_t)f[j] * r, r);
         float y[E + 1];
         sum_parts<E + (AD ? 1 : 0), AD ? 4 : 8>(P, 0, m, f, y, tag);
+        unsigned long long *sw = (it == 0 && lane == 0) ? st : nullptr;  // first row's sub-steps
+        stamp_at(sw, 9);
         float u[MAX_RANK];
         if (AD) share_u(y[E], 0, u);
 #pragma unroll
@@ -518,6 +528,7 @@ __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, 
                 y[j + E / 2] = rbf(__fadd_rn(__fmul_rn(c, cs.x), __fmul_rn(a, cs.y)));
             }
         }
+        stamp_at(sw, 10);
         if (kind == 0) {
             bf16 *dst = P.q + ((size_t)m * dm.Hq + head) * DH;
 #pragma unroll
@@ -534,13 +545,14 @@ __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, 
 #pragma unroll
             for (int j = 0; j < E; ++j) dst[lane + 32 * j] = f2bf(y[j]);
         }
+        stamp_at(sw, 11);
     }
 }
 
 // o or down tile: adapter delta, residual add into h, per-tile sum of squares
 template <bool AD>
 __device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int layer, int tile, int cw, int lane, int m0,
-                                             int mstep, uint32_t tag) {
+                                             int mstep, uint32_t tag, unsigned long long *st) {
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r, H = dm.H, nt = H / TILE_ROWS;
     const bf16 *lb = P.lora_b[lin] + (size_t)layer * P.lb_stride[lin];
@@ -561,6 +573,8 @@ __device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int lay
         }
         f[4] = P.n_main[lin] + (lane < r ? lane : 0);
         sum_parts<AD ? 5 : 4, AD ? 4 : 8>(P, lin, m, f, acc, tag);
+        unsigned long long *sw = (cw == 0 && m == m0 && lane == 0) ? st : nullptr;  // first row's sub-steps
+        stamp_at(sw, 9);
         float u[MAX_RANK];
         if (AD) share_u(acc[4], 0, u);
         float v[4];
@@ -570,15 +584,17 @@ __device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int lay
             v[e] = rbf(__fadd_rn(hv[e], rbf(acc[e])));
             P.h[(size_t)m * H + f[e]] = f2bf(v[e]);
         }
+        stamp_at(sw, 10);
         const float s = tile_sumsq(v);
         if (lane == 0) P.ss[(size_t)m * nt + tile] = s;
+        stamp_at(sw, 11);
     }
 }
 
 // gate|up tile (rows 0-63 gate features 64t.., rows 64-127 up features 64t..): SiLU(gate)*up
 template <bool AD>
 __device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, int cw, int lane, int m0, int mstep,
-                                      uint32_t tag) {
+                                      uint32_t tag, unsigned long long *st) {
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r, I = dm.I;
     const bf16 *lb = P.lora_b[2] + (size_t)layer * P.lb_stride[2];
@@ -598,6 +614,8 @@ __device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, i
                           tile * TILE_ROWS + 96 + lane, P.n_main[2] + (lane < 2 * r ? lane : 0)};
         float ug[MAX_RANK], uu[MAX_RANK], s[5];
         sum_parts<AD ? 5 : 4, 2>(P, 2, m, f, s, tag);
+        unsigned long long *sw = (cw == 0 && m == m0 && lane == 0) ? st : nullptr;  // first row's sub-steps
+        stamp_at(sw, 9);
         if (AD) {
             share_u(s[4], 0, ug);
             share_u(s[4], r, uu);
@@ -619,6 +637,7 @@ __device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, i
             if ((lane & 1) == 0)
                 st_relaxed_u64(P.act + ((size_t)m * I + a) / 2, ((unsigned long long)tag << 32) | (hi << 16) | bits);
         }
+        stamp_at(sw, 11);
     }
 }
 
@@ -723,6 +742,7 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
             qa[ks][2] = val0 ? __ldcg(reinterpret_cast<const unsigned *>(q0 + c + 8)) : 0u;
             qa[ks][3] = val1 ? __ldcg(reinterpret_cast<const unsigned *>(q1 + c + 8)) : 0u;
         }
+        unsigned long long *sw = (unit == 0 && lane == 0) ? stamp : nullptr;  // first unit's sub-steps
         float sc[NT][4];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
@@ -742,6 +762,7 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
                 mma_m16n8k16_bf16(sc[nt], qa[ks + 1], b2, b3);
             }
         }
+        stamp_at(sw, 9);
         const int qp0 = L + i0, qp1 = L + i1;
         // last visible key of each row: causal rows see up to themselves; in the draft the
         // block's mask rows (i >= 1) also see the rest of the block
@@ -793,6 +814,7 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
             pa[kstep][2] = pack_half2(sc[2 * kstep + 1][0], sc[2 * kstep + 1][1]);
             pa[kstep][3] = pack_half2(sc[2 * kstep + 1][2], sc[2 * kstep + 1][3]);
         }
+        stamp_at(sw, 10);
         const int nsa = P.att_splits_alloc;
         const int sub = s * ATT_SUBS + half;  // index of this partial result
         float *dst0 = val0 ? P.o_part + (((size_t)(bl * R + i0) * dm.Hq + h0) * nsa + sub) * DH : nullptr;
@@ -829,12 +851,14 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
             P.ml_part[((size_t)(bl * R + i0) * dm.Hq + h0) * nsa + sub] = make_float2(m0, l0);
         if (val1 && tq == 0)
             P.ml_part[((size_t)(bl * R + i1) * dm.Hq + h1) * nsa + sub] = make_float2(m1, l1);
+        stamp_at(sw, 11);
     }
 }
 
 // merge the splits of (row, head) in split order; splits where the row saw no key are skipped
 template <int DH>
-__device__ __noinline__ void attn_combine(const MKParams &P, int bl, int g, int cw, int lane, int p0, int pstep) {
+__device__ __noinline__ void attn_combine(const MKParams &P, int bl, int g, int cw, int lane, int p0, int pstep,
+                                          unsigned long long *st) {
     const Dims &dm = P.dm;
     const int R = P.pd.R, grp = dm.Hq / dm.Hkv;
     const int b = P.pd.b0 + bl;
@@ -862,6 +886,7 @@ __device__ __noinline__ void attn_combine(const MKParams &P, int bl, int g, int 
 #pragma unroll
         for (int u = 0; u < NB; ++u)
             if (v[u].y > 0.f) mx = fmaxf(mx, v[u].x);
+        if (cw == 0 && it == p0 && lane == 0) stamp_at(st, 12);
         for (int s0 = NB; s0 < nv; s0 += NB) {  // long contexts only: NB statistics per round
             float2 w[NB];
 #pragma unroll
@@ -1097,7 +1122,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
         // ---------------- compute group (warps 2-7)
         const int ct = tid - 64, cw = warp - 2;
         uint32_t li = 0, ai = 0, l8 = 0;
-        unsigned long long *tr = P.trace ? P.trace + 8ull * P.cta_off[blockIdx.x] : nullptr;
+        unsigned long long *tr = P.trace ? P.trace + (size_t)MK_STAMPS * P.cta_off[blockIdx.x] : nullptr;
         // the attention pages are requested by thread CT_PAGES while thread 0 polls the item's
         // inputs; att_pend (that thread only): pages requested for a split that has not waited
         bool att_pend = false;
@@ -1105,8 +1130,8 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
             const MKItem it = my[i];
             if (tr && ct == 0) {
                 const unsigned long long now = globaltimer_ns();
-                if (i > 0) tr[8 * (i - 1) + 3] = now;
-                tr[8 * i] = now;
+                if (i > 0) tr[MK_STAMPS * (i - 1) + 3] = now;
+                tr[MK_STAMPS * i] = now;
             }
             const bool att_active = it.op == MK_ATTN && it.c * ATT_SPLIT < P.L[P.pd.b0 + it.a] + P.pd.R;
             if (att_active && ct == CT_PAGES) {
@@ -1119,7 +1144,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
             if (ct == 0) s_flag = wait_deps(P, it) ? 1 : 0;
             bar_compute();
             if (!s_flag) break;
-            if (tr && ct == 0) tr[8 * i + 1] = tr[8 * i + 2] = globaltimer_ns();
+            if (tr && ct == 0) tr[MK_STAMPS * i + 1] = tr[MK_STAMPS * i + 2] = globaltimer_ns();
             if (it.op == MK_EMBED) {
                 do_embed(P, it.a, cw, lane);
                 bar_compute();
@@ -1150,14 +1175,15 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                         if (nb1) fence_proxy_async_global();
                         mbar_arrive_expect_tx(&att_bar, nb1);
                         if (nb1) attn_pages(P, it.layer, bl, g, s, 1, uni, &att_bar, true);
+                        if (tr) tr[MK_STAMPS * i + 8] = globaltimer_ns();
                     }
-                    unsigned long long *st = tr ? tr + 8 * i : nullptr;
+                    unsigned long long *st = tr ? tr + MK_STAMPS * i : nullptr;
                     attn_split<DH, DRAFT>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st);
                     ++ai;
                     att_pend = false;
                 }
                 bar_compute();
-                if (tr && ct == 0) tr[8 * i + 2] = globaltimer_ns();
+                if (tr && ct == 0) tr[MK_STAMPS * i + 2] = globaltimer_ns();
                 // merge: when the (sequence, head)'s splits fit on distinct CTAs, every split waits for
                 // the others and merges pairs s, s + nsplit, ...; otherwise the last one merges all
                 int *c = ctr(P, it.layer, P.cl.att + bl * P.dm.Hkv + g);
@@ -1173,42 +1199,43 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                         s_ok = 1;
                     }
                 }
-                if (tr && ct == 0) tr[8 * i + 6] = tr[8 * i + 7] = globaltimer_ns();
+                if (tr && ct == 0) tr[MK_STAMPS * i + 6] = tr[MK_STAMPS * i + 7] = globaltimer_ns();
                 bar_compute();
                 if (!s_ok) break;
                 if (s_red) {
                     const int p0 = shared_merge ? s : 0, pstep = shared_merge ? nsp : 1;
-                    attn_combine<DH>(P, bl, g, cw, lane, p0, pstep);
+                    attn_combine<DH>(P, bl, g, cw, lane, p0, pstep, tr ? tr + MK_STAMPS * i : nullptr);
                     bar_compute();
                     if (ct == 0) red_release_add(c, 1);
-                    if (tr && ct == 0) tr[8 * i + 7] = globaltimer_ns();
+                    if (tr && ct == 0) tr[MK_STAMPS * i + 7] = globaltimer_ns();
                 }
             } else {
                 // ---- linear slice item: stage activations, MMA (warp 1), epilogue, split reduction
                 const int lin = it.lin, l = it.layer, t = it.a, s = it.b;
                 const int na = P.katoms[lin];
+                unsigned long long *st_i = tr ? tr + MK_STAMPS * i : nullptr;
                 if (na <= HALF_ATOMS) {
                     if (lin == 3)
-                        build_b_act(P, s, uni, ct, s_tag + l);
+                        build_b_act(P, s, uni, ct, s_tag + l, st_i);
                     else
-                        build_b(P, lin, l, s, uni, s_rms, ct, 0, na, true);
+                        build_b(P, lin, l, s, uni, s_rms, ct, 0, na, true, st_i);
                     fence_proxy_async();
                     bar_compute();
                     if (ct == 0) mbarrier_arrive_one(&b_full[0]);
                 } else if (P.b_dbl) {
                     // wide slice, both halves fit: the first half's MMAs run while the second is staged
-                    build_b(P, lin, l, s, uni, s_rms, ct, 0, HALF_ATOMS, true);
+                    build_b(P, lin, l, s, uni, s_rms, ct, 0, HALF_ATOMS, true, st_i);
                     fence_proxy_async();
                     bar_compute();
                     if (ct == 0) mbarrier_arrive_one(&b_full[0]);
                     build_b(P, lin, l, s, uni + (size_t)HALF_ATOMS * P.bn * 128, s_rms, ct, HALF_ATOMS,
-                            na - HALF_ATOMS, false);
+                            na - HALF_ATOMS, false, nullptr);
                     fence_proxy_async();
                     bar_compute();
                     if (ct == 0) mbarrier_arrive_one(&b_full[1]);
                 } else {
                     // operand in two rounds through the same area
-                    build_b(P, lin, l, s, uni, s_rms, ct, 0, HALF_ATOMS, true);
+                    build_b(P, lin, l, s, uni, s_rms, ct, 0, HALF_ATOMS, true, st_i);
                     fence_proxy_async();
                     bar_compute();
                     if (ct == 0) {
@@ -1217,19 +1244,19 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                     }
                     bar_compute();
                     if (!s_ok) break;
-                    build_b(P, lin, l, s, uni, s_rms, ct, HALF_ATOMS, na - HALF_ATOMS, false);
+                    build_b(P, lin, l, s, uni, s_rms, ct, HALF_ATOMS, na - HALF_ATOMS, false, nullptr);
                     fence_proxy_async();
                     bar_compute();
                     if (ct == 0) mbarrier_arrive_one(&b_full[1]);
                 }
                 if (na > HALF_ATOMS) ++l8;
-                if (tr && ct == 0) tr[8 * i + 4] = globaltimer_ns();
+                if (tr && ct == 0) tr[MK_STAMPS * i + 4] = globaltimer_ns();
                 const bool lt = t >= P.n_main[lin] / TILE_ROWS;
                 const int rows_valid = lt ? P.lora_rows[lin] : TILE_ROWS;
                 if (warp >= 4) {
                     const int quarter = warp - 4;
                     const bool have = mbar_wait_mk(&acc_full, li & 1, P, DEV_TIMEOUT_MMA);
-                    if (tr && warp == 4 && lane == 0) tr[8 * i + 5] = globaltimer_ns();
+                    if (tr && warp == 4 && lane == 0) tr[MK_STAMPS * i + 5] = globaltimer_ns();
                     tc_fence_after();
                     if (have) {
                         const int row = quarter * 32 + lane;
@@ -1252,25 +1279,25 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 }
                 ++li;
                 bar_compute();
-                if (tr && ct == 0) tr[8 * i + 2] = globaltimer_ns();
+                if (tr && ct == 0) tr[MK_STAMPS * i + 2] = globaltimer_ns();
                 // The tile's slices are consecutive items of the round-robin schedule, so they sit on
                 // distinct CTAs that all reach them: each CTA stores its tagged slice partials, then
                 // reduces rows s, s + ks, ... of the tile (s = its slice), reading the other slices'
                 // partials as they arrive. The adapter tile's partials are summed by the main tiles'
                 // reducers themselves.
                 const int ks = P.ks[lin];
-                if (tr && ct == 0) tr[8 * i + 6] = globaltimer_ns();
+                if (tr && ct == 0) tr[MK_STAMPS * i + 6] = globaltimer_ns();
                 if (lt) {
-                    if (tr && ct == 0) tr[8 * i + 7] = globaltimer_ns();
+                    if (tr && ct == 0) tr[MK_STAMPS * i + 7] = globaltimer_ns();
                     continue;
                 }
                 const uint32_t tag = s_tag + l;
                 if (lin == 0) {
-                    reduce_qkv<DH, DRAFT>(P, l, t, cw, lane, s, ks, tag);
+                    reduce_qkv<DH, DRAFT>(P, l, t, cw, lane, s, ks, tag, st_i);
                 } else if (lin == 2)
-                    reduce_gu<DRAFT>(P, l, t, cw, lane, s, ks, tag);
+                    reduce_gu<DRAFT>(P, l, t, cw, lane, s, ks, tag, st_i);
                 else
-                    reduce_residual<DRAFT>(P, lin, l, t, cw, lane, s, ks, tag);
+                    reduce_residual<DRAFT>(P, lin, l, t, cw, lane, s, ks, tag, st_i);
                 bar_compute();
                 if (ct == 0) {
                     // one release per reduction, on the counter its consumers poll
@@ -1282,10 +1309,10 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                         for (int g = g0; g <= g1; ++g) red_release_add(ctr(P, l, P.cl.att_in + g), 1);
                     }
                 }
-                if (tr && ct == 0) tr[8 * i + 7] = globaltimer_ns();
+                if (tr && ct == 0) tr[MK_STAMPS * i + 7] = globaltimer_ns();
             }
         }
-        if (tr && ct == 0 && n_my > 0) tr[8 * (n_my - 1) + 3] = globaltimer_ns();
+        if (tr && ct == 0 && n_my > 0) tr[MK_STAMPS * (n_my - 1) + 3] = globaltimer_ns();
         if (ct == CT_PAGES && att_pend) {
             // the pass ended before the split waited for its pages: complete the phase's arrival
             // and let the copies land (bounded) before the shared memory is released

@@ -289,7 +289,7 @@ size_t layout(pbd_ctx *c, void *base) {
     c->ml_part = (float2 *)bp.take(sizeof(float2) * (size_t)RA * Hq * c->n_splits * ATT_SUBS);
     c->tile_max = (float *)bp.take(sizeof(float) * (size_t)(V / TILE_ROWS) * c->ro_alloc);
     c->tile_arg = (int *)bp.take(sizeof(int) * (size_t)(V / TILE_ROWS) * c->ro_alloc);
-    c->trace = (unsigned long long *)bp.take(sizeof(unsigned long long) * 8 * c->items_cap);
+    c->trace = (unsigned long long *)bp.take(sizeof(unsigned long long) * MK_STAMPS * c->items_cap);
     return bp.off + ALIGN;
 }
 
@@ -1094,12 +1094,12 @@ pbd_status pbd_trace_pass(pbd_ctx *c, int32_t kind, int32_t *h_items, uint64_t *
     if ((int)items.size() > cap) return fail(c, PBD_ERR_CAPACITY, "%zu items exceed cap %d", items.size(), cap);
     CK(launch_build_ids(pd, kind == PK_DRAFT ? 0 : (kind == PK_VERIFY ? 1 : 2), c->s.pending, c->draft_ids, c->D,
                         c->ids, c->st));
-    CK(cudaMemsetAsync(c->trace, 0, sizeof(unsigned long long) * 8 * items.size(), c->st));
+    CK(cudaMemsetAsync(c->trace, 0, sizeof(unsigned long long) * MK_STAMPS * items.size(), c->st));
     CK(cudaMemsetAsync(c->cnt, 0, sizeof(int) * (size_t)(c->cl.total + 1), c->st));
     MKLaunch L = make_launch(c, pd, kind);
     L.trace = c->trace;
     CK(launch_pass_kernel(L, c->st));
-    CK(cudaMemcpyAsync(h_trace, c->trace, sizeof(unsigned long long) * 8 * items.size(), cudaMemcpyDeviceToHost,
+    CK(cudaMemcpyAsync(h_trace, c->trace, sizeof(unsigned long long) * MK_STAMPS * items.size(), cudaMemcpyDeviceToHost,
                        c->st));
     CK(cudaStreamSynchronize(c->st));
     for (size_t i = 0; i < items.size(); ++i) {

@@ -67,6 +67,16 @@ struct Partials {
 
 enum MKOp : uint8_t { MK_EMBED = 0, MK_LINEAR = 1, MK_ATTN = 2, MK_FINAL = 3 };
 
+// Timestamps per item recorded by a traced pass (%globaltimer ns; 0 = not reached):
+//   0 start, 1 inputs ready, 2 work done, 3 end (next item's start);
+//   linear items: 4 operand staged, 5 accumulator ready, 6 partials stored, 7 reduced,
+//     8 norm scales ready (RMSNorm inputs) or act words valid (down), 9 first reduced row's
+//     partial sums present, 10 its outputs computed, 11 reduction's stores issued;
+//   attention items: 4 K/V pages landed, 5 V converted, 6 counted (all splits stored), 7 merged,
+//     8 block pages requested, 9 q fragments loaded, 10 softmax done, 11 partials stored,
+//     12 merge inputs loaded.
+constexpr int MK_STAMPS = 16;
+
 // One work item of a pass.  MK_LINEAR: lin (0 q|k|v, 1 o, 2 gate|up, 3 down), a = row tile
 // (the adapter tile is the last one), b = 256-wide K slice.  MK_ATTN: a = sequence in the pass,
 // b = KV head, c = 128-key split.  MK_EMBED: a = row.  MK_FINAL: a = read-out index, b = row.

@@ -21,6 +21,7 @@ PBD_OK = 0
 STATUS_NAMES = {0: "PBD_OK", 1: "PBD_ERR_INVALID_ARG", 2: "PBD_ERR_WORKSPACE", 3: "PBD_ERR_CAPACITY",
                 4: "PBD_ERR_STATE", 5: "PBD_ERR_CUDA", 6: "PBD_ERR_DEVICE"}
 LINEARS = ("q", "k", "v", "o", "gate", "up", "down")
+TRACE_STAMPS = 16  # timestamps per work item of pbd_trace_pass
 
 
 class PbdError(RuntimeError):
@@ -418,13 +419,13 @@ class Engine:
         return float(ms[0]), float(ms[1]), float(ms[2]), float(ms[3]), int(launches[0])
 
     def pbd_trace_pass(self, kind: int, cap: int = 400000):
-        """(items [n, 4] int32 {op|lin<<8|layer<<16, a, b, c}, stamps [n, 8] uint64 ns) of one traced pass."""
+        """(items [n, 4] int32 {op|lin<<8|layer<<16, a, b, c}, stamps [n, 16] uint64 ns) of one traced pass."""
         items = np.zeros(cap * 4, np.int32)
-        tr = np.zeros(cap * 8, np.uint64)
+        tr = np.zeros(cap * TRACE_STAMPS, np.uint64)
         n = np.zeros(1, np.int32)
         self._call(self.lib.pbd_trace_pass, kind, items.ctypes.data, tr.ctypes.data, cap, n.ctypes.data)
         k = int(n[0])
-        return items[: 4 * k].reshape(k, 4), tr[: 8 * k].reshape(k, 8)
+        return items[: 4 * k].reshape(k, 4), tr[: TRACE_STAMPS * k].reshape(k, TRACE_STAMPS)
 
     def pbd_check_stalled_pass(self):
         """(status, device code) of a verify pass missing one item (see include/pbd.h)."""

@@ -38,8 +38,8 @@ def summarize(items, tr):
         out["phases"][name] = {"items": int(sel.sum()), "wait_us_med": float(np.median(wait)),
                                "work_us_med": float(np.median(work)), "post_us_med": float(np.median(post)),
                                "item_us_max": float((t[sel, 3] - t[sel, 0]).max())}
-        # sub-stamps 4..7 (0 = not reached): linear = operand staged, accumulator ready, counted,
-        # reduced; attention = K/V landed, V converted, counted, merged
+        # sub-stamps 4..7 (0 = not reached): linear = operand staged, accumulator ready, partials
+        # stored, reduced; attention = K/V landed, V converted, all splits stored, merged
         sub = {}
         labels = (("staged", "acc_ready", "counted", "reduced") if name not in ("attn",)
                   else ("landed", "converted", "counted", "merged"))
@@ -47,6 +47,16 @@ def summarize(items, tr):
             ok = sel & (tr[:, 4 + j] > 0)
             if ok.any():
                 sub[lab + "_us_med"] = float(np.median(t[ok, 4 + j] - t[ok, 1]))
+        # finer sub-steps 8..12 (present when the stamps are 16 wide), as means: the timer ticks
+        # in steps of a few hundred ns, so means over many items resolve finer than medians
+        labels2 = (("norm_or_act_ready", "first_row_summed", "first_row_computed", "reduce_stored")
+                   if name not in ("attn",) else
+                   ("block_requested", "scores_done", "softmax_done", "partials_stored", "merge_loaded"))
+        if tr.shape[1] >= 16:
+            for j, lab in enumerate(labels2):
+                ok = sel & (tr[:, 8 + j] > 0)
+                if ok.any():
+                    sub[lab + "_us_mean"] = float(np.mean(t[ok, 8 + j] - t[ok, 1]))
         if sub:
             out["phases"][name]["since_deps"] = sub
         ends[name] = {int(l): float(t[sel & (layer == l), 3].max()) for l in np.unique(layer[sel])}

@@ -204,7 +204,7 @@ def test_pass_timing_and_trace_entry_points(env):
     """pbd_time_pass and pbd_trace_pass run a pass on a prefilled context without advancing it:
     positive times and byte counts, every scheduled item traced once with ordered stamps, and
     the generation state unchanged afterwards."""
-    eng, prompt = env["eng"], env["prompts"][1]
+    eng, prompt, pbd = env["eng"], env["prompts"][1], env["pbd"]
     eng.pbd_prefill([prompt], max_new=32)
     before = [np.asarray(x).copy() for x in eng.pbd_get_state()]
     for kind in (0, 1, 2):
@@ -212,7 +212,7 @@ def test_pass_timing_and_trace_entry_points(env):
         assert ms > 0 and nbytes > 0
         items, st = eng.pbd_trace_pass(kind)
         assert len(items) == len(st) > 0
-        assert st.shape[1] == 8
+        assert st.shape[1] == pbd.TRACE_STAMPS == 16
         ops = items[:, 0] & 0xFF
         assert set(np.unique(ops)) <= {0, 1, 2, 3}
         # start <= inputs ready <= end for every item (all stamps from one global clock)
