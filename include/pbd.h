@@ -213,8 +213,11 @@ pbd_status pbd_check_stalled_pass(pbd_ctx *ctx, int32_t *h_device_code);
  * of the schedule's properties).  For a generation of `batch` prompts of h_prompt_lens tokens
  * and a budget of max_new tokens under cfg (whose draft variant applies to kind 0), returns the
  * items of a draft (kind 0), verify (1) or plain-decoding (2) pass dealt round-robin over `grid`
- * CTAs: h_items[4 i..4 i+3] = {op | lin << 8 | layer << 16, a, b, c} (op 0 embedding row, 1
- * linear slice, 2 attention split, 3 final norm; see pbd_trace_pass), grouped by CTA with CTA
+ * CTAs: h_items[8 i..8 i+7] = {op | lin << 8 | layer << 16, a, b, c, wait counter, wait target,
+ * release counter 0, release counter 1} (op 0 embedding row, 1 linear slice, 2 attention split,
+ * 3 final norm; see pbd_trace_pass; the item waits until the pass counter `wait counter` (-1:
+ * none) reaches `wait target`, and adds one to each release counter >= 0 once its result is
+ * stored), grouped by CTA with CTA
  * k's items at [h_cta_off[k], h_cta_off[k + 1]) (h_cta_off has grid + 1 entries; CTA k takes
  * the topologically ordered list's items k, k + grid, ...).  *h_n is the item count; at most
  * `cap` items are written (PBD_ERR_CAPACITY beyond).  Errors: PBD_ERR_INVALID_ARG (bad config or

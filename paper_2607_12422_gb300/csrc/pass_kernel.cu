@@ -136,16 +136,20 @@ __device__ __forceinline__ void stamp_at(unsigned long long *st, int k) {
     if (st) st[k] = globaltimer_ns();
 }
 
-__device__ __forceinline__ void raise_abort(const MKParams &P, int code) {
+// Code size matters here: the compute warps walk every kind of item each layer, and code the
+// SM's instruction caches cannot hold streams from L2 at several cycles per instruction.  Wait
+// loops, error paths and rarely taken branches are therefore kept out of line and not unrolled.
+__device__ __noinline__ void raise_abort(const MKParams &P, int code) {
     latch_error(P.status, code);
     atomicExch(P.abort, 1);
 }
 
 // one thread: wait until *c >= target (bounded)
-__device__ bool spin_until(const int *c, int target, const MKParams &P) {
+__device__ __noinline__ bool spin_until(const int *c, int target, const MKParams &P) {
     if (ld_acquire(c) >= target) return true;
     const uint64_t t0 = globaltimer_ns();
     for (;;) {
+#pragma unroll 1
         for (int i = 0; i < 8; ++i) {
             if (ld_acquire(c) >= target) return true;
             __nanosleep(40);
@@ -160,19 +164,18 @@ __device__ bool spin_until(const int *c, int target, const MKParams &P) {
 
 // bounded mbarrier wait that does not give up on abort: the pass is ending and its asynchronous
 // copies and MMAs must land before the CTA releases its shared memory and TMEM
-__device__ __forceinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
+__device__ __noinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
     const uint32_t a = smem_u32(bar);
     const uint64_t t0 = globaltimer_ns();
     while (!mbar_try_wait(a, parity) && globaltimer_ns() - t0 < WAIT_LIMIT_NS) {
     }
 }
 
-// bounded mbarrier wait that also gives up when the pass is aborted
-__device__ bool mbar_wait_mk(uint64_t *bar, uint32_t parity, const MKParams &P, int code) {
-    const uint32_t a = smem_u32(bar);
-    if (mbar_try_wait(a, parity)) return true;
+// bounded mbarrier wait that also gives up when the pass is aborted (slow path out of line)
+__device__ __noinline__ bool mbar_wait_slow(uint32_t a, uint32_t parity, const MKParams &P, int code) {
     const uint64_t t0 = globaltimer_ns();
     for (;;) {
+#pragma unroll 1
         for (int i = 0; i < 16; ++i)
             if (mbar_try_wait(a, parity)) return true;
         if (aborted(P)) return false;
@@ -181,6 +184,10 @@ __device__ bool mbar_wait_mk(uint64_t *bar, uint32_t parity, const MKParams &P, 
             return false;
         }
     }
+}
+__device__ __forceinline__ bool mbar_wait_mk(uint64_t *bar, uint32_t parity, const MKParams &P, int code) {
+    const uint32_t a = smem_u32(bar);
+    return mbar_try_wait(a, parity) || mbar_wait_slow(a, parity, P, code);
 }
 
 __device__ __forceinline__ int *ctr(const MKParams &P, int layer, int off) {
@@ -259,52 +266,59 @@ __device__ __forceinline__ void share_u(float lane_sum, int base, float (&u)[MAX
     for (int j = 0; j < MAX_RANK; ++j) u[j] = __shfl_sync(0xffffffffu, a, base + j);
 }
 
-// Sums of the K-slice partials of E features of row m, slices added in order; loads go out
-// in batches of S slices (every load of a batch in flight before the first add).
-// Each partial is one 64-bit word, the fp32 value and the tag of the (pass, layer) that stored
-// it, written and read with single-copy-atomic accesses: a word carrying this layer's tag holds
-// this layer's value, so the sum polls the words themselves instead of a completion counter.
-// Words still carrying an older tag are read again (bounded; on timeout or abort the pass is lost).
-template <int E, int S>
-__device__ __forceinline__ void sum_parts(const MKParams &P, int lin, int m, const int *f, float *out, uint32_t tag) {
+// Feature offsets (from a lane's first feature f0) of the four partial sums a lane reduces: two
+// pairs of adjacent features, the second pair at f0 + OFF2 (2 for four consecutive features,
+// 64 for gate|up: a gate pair and the up pair of the same act features).
+// Sums of the K-slice partials of row m: out[0..3] for features f0, f0 + 1, f0 + OFF2, f0 + OFF2 + 1
+// and, when X, out[4] for feature fx; slices added in order, loads in batches of S slices (every
+// load of a batch in flight before the first add).  Each partial is one 64-bit word, the fp32
+// value and the tag of the (pass, layer) that stored it, written and read with single-copy-atomic
+// accesses: a word carrying this layer's tag holds this layer's value, so the sum polls the words
+// themselves instead of a completion counter.  A batch with a word still carrying an older tag is
+// read again (bounded; on timeout or abort the pass is lost).  One copy of the load code serves
+// the first read and the re-reads, which keeps the function small.
+template <int OFF2, bool X, int S>
+__device__ __forceinline__ void sum_parts(const MKParams &P, int lin, int m, int f0, int fx, float *out, uint32_t tag) {
+    constexpr int EX = 4 + (X ? 1 : 0);
     const int nt = P.n_main[lin] + P.lora_rows[lin];
     const unsigned long long *p = P.part[lin] + (size_t)m * nt;
     const size_t stride = (size_t)P.part_rows * nt;
     const int ks = P.ks[lin];
+    const unsigned long long none = (unsigned long long)tag << 32;
+#pragma unroll 1
     for (int s0 = 0; s0 < ks; s0 += S) {
-        unsigned long long v[E][S];
+        unsigned long long v[EX][S];
+        uint64_t t0 = 0;
+#pragma unroll 1
+        for (int round = 0;; ++round) {
 #pragma unroll
-        for (int s = 0; s < S; ++s)
+            for (int s = 0; s < S; ++s) {
+                const unsigned long long *ps = p + (size_t)(s0 + s) * stride;
+                if (s0 + s < ks) {
+                    ld_relaxed_2u64(ps + f0, v[0][s], v[1][s]);
+                    ld_relaxed_2u64(ps + f0 + OFF2, v[2][s], v[3][s]);
+                    if (X) v[EX - 1][s] = ld_relaxed_u64(ps + fx);
+                } else {
 #pragma unroll
-            for (int e = 0; e < E; ++e)
-                v[e][s] = s0 + s < ks ? ld_relaxed_u64(p + (s0 + s) * stride + f[e]) : (unsigned long long)tag << 32;
-        bool stale = false;
-#pragma unroll
-        for (int s = 0; s < S; ++s)
-#pragma unroll
-            for (int e = 0; e < E; ++e) stale |= (uint32_t)(v[e][s] >> 32) != tag;
-        if (stale) {
-            const uint64_t t0 = globaltimer_ns();
-            for (int round = 1; stale; ++round) {
-                __nanosleep(32);
-                stale = false;
-#pragma unroll
-                for (int s = 0; s < S; ++s)
-#pragma unroll
-                    for (int e = 0; e < E; ++e)
-                        if ((uint32_t)(v[e][s] >> 32) != tag) {
-                            v[e][s] = ld_relaxed_u64(p + (s0 + s) * stride + f[e]);
-                            stale |= (uint32_t)(v[e][s] >> 32) != tag;
-                        }
-                // the abort flag and the time limit every 8 rounds (each check is an L2 round trip)
-                if (stale && (round & 7) == 0 && (aborted(P) || globaltimer_ns() - t0 > WAIT_LIMIT_NS)) {
-                    if (!aborted(P)) raise_abort(P, DEV_TIMEOUT_DEP);
-                    break;
+                    for (int e = 0; e < EX; ++e) v[e][s] = none;
                 }
+            }
+            bool stale = false;
+#pragma unroll
+            for (int s = 0; s < S; ++s)
+#pragma unroll
+                for (int e = 0; e < EX; ++e) stale |= (uint32_t)(v[e][s] >> 32) != tag;
+            if (!stale) break;
+            // the abort flag and the time limit every 8 rounds (each check is an L2 round trip)
+            if (round == 0) t0 = globaltimer_ns();
+            __nanosleep(32);
+            if ((round & 7) == 7 && (aborted(P) || globaltimer_ns() - t0 > WAIT_LIMIT_NS)) {
+                if (!aborted(P)) raise_abort(P, DEV_TIMEOUT_DEP);
+                break;
             }
         }
 #pragma unroll
-        for (int e = 0; e < E; ++e) {
+        for (int e = 0; e < EX; ++e) {
 #pragma unroll
             for (int s = 0; s < S; ++s) {
                 if (s0 + s >= ks) break;
@@ -347,58 +361,55 @@ __device__ __noinline__ void do_embed(const MKParams &P, int m, int cw, int lane
     }
 }
 
-// Activation tile of one linear item in the 128-byte swizzle layout: atom j (K columns
-// 64j..64j+63 of the slice) holds row m at m*128 bytes, 16-byte chunk c at (c ^ (m & 7)) * 16.
-// Row m of the q|k|v and gate|up inputs is RMSNorm(h_m) * gain, computed here on the fly.
+// Activation tile of one linear item in the 128-byte swizzle layout: four atoms (K columns
+// 64j..64j+63 of the slice, starting a0 atoms into it) hold row m at m*128 bytes, 16-byte chunk c
+// at (c ^ (m & 7)) * 16.  The chunks are copied straight into place with cp.async (one L2 round
+// trip whatever the row count).  Rows of the q|k|v and gate|up inputs are then normalised in
+// place: bf16(g * bf16(h * rs)), the product with the gain taken in bf16x2 (the exact product of
+// two bf16 numbers rounded once to nearest even, as fp32 and then rounding gives).  A row has
+// 32 chunks of 8 elements; thread ct handles chunks ct, ct + 192, ..., so its chunk column
+// (ct % 32), and with it its gain chunk, is the same for all of them.
 __device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int slice, uint8_t *sb, float *s_rms, int ct,
-                                     int a0, int na, bool need_rms, unsigned long long *st) {
-    constexpr int U = 4;  // chunks in flight per thread
+                                     int a0, bool need_rms, unsigned long long *st) {
     const int M = P.pd.M;
-    const int k0 = (slice * P.katoms[lin] + a0) * KT;
-    const int cpr = na * (KT / 8);  // 16-byte chunks per row
-    const bool norm = (lin == 0 || lin == 2);
-    const bf16 *gain = lin == 0 ? P.attn_norm + (size_t)layer * P.dm.H : P.mlp_norm + (size_t)layer * P.dm.H;
-    const bf16 *src = norm ? P.h : P.attn;  // the down projection's operand: build_b_act
-    const int ld = norm ? P.dm.H : (lin == 1 ? P.dm.Hq * P.dm.d : P.dm.I);
-    const int chunks = M * cpr;
-    uint4 xv[U], gv[U];
-    auto issue = [&](int q0) {
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int q = q0 + u * CT;
-            if (q < chunks) {
-                const int m = q / cpr, c = q % cpr;
-                xv[u] = __ldcg(reinterpret_cast<const uint4 *>(src + (size_t)m * ld + k0 + c * 8));
-                if (norm) gv[u] = __ldg(reinterpret_cast<const uint4 *>(gain + k0 + c * 8));
-            }
-        }
-    };
-    // the first chunks are in flight while the rows' norm scales are computed
-    issue(ct);
-    if (norm && need_rms) {
+    const bool norm = lin != 1;
+    const bf16 *src = norm ? P.h : P.attn;  // (the down projection's operand: build_b_act)
+    const int ld = norm ? P.dm.H : P.dm.Hq * P.dm.d;
+    const int chunks = M * 32, c = ct & 31;
+    const size_t col = (size_t)(slice * P.katoms[lin] + a0) * KT + c * 8;
+    uint8_t *dst_c = sb + (size_t)(c >> 3) * P.bn * 128 + ((c & 7) << 4);
+#pragma unroll 1
+    for (int q = ct; q < chunks; q += CT) {
+        const int m = q >> 5;
+        cp_async16(dst_c + m * 128 - ((c & 7) << 4) + (((c & 7) ^ (m & 7)) << 4), src + (size_t)m * ld + col);
+    }
+    cp_async_commit();
+    if (!norm) {
+        cp_async_wait_all();
+        return;
+    }
+    const uint4 gv = __ldg(reinterpret_cast<const uint4 *>((lin == 0 ? P.attn_norm : P.mlp_norm) + (size_t)layer * P.dm.H + col));
+    if (need_rms)  // while the copies are in flight
         for (int m = ct; m < M; m += CT) s_rms[m] = row_rms(P, m);
+    cp_async_wait_all();
+    if (need_rms) {
         bar_compute();
         if (ct == 0) stamp_at(st, 8);
     }
-    for (int q0 = ct; q0 < chunks; q0 += U * CT) {
-        if (q0 != ct) issue(q0);
+    const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(&gv);
+#pragma unroll 1
+    for (int q = ct; q < chunks; q += CT) {
+        const int m = q >> 5;
+        uint4 *p = reinterpret_cast<uint4 *>(dst_c + m * 128 - ((c & 7) << 4) + (((c & 7) ^ (m & 7)) << 4));
+        uint4 val = *p;
+        __nv_bfloat162 *v2 = reinterpret_cast<__nv_bfloat162 *>(&val);
+        const float rs = s_rms[m];
 #pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int q = q0 + u * CT;
-            if (q >= chunks) break;
-            const int m = q / cpr, c = q % cpr;
-            const int atom = c >> 3, cc = c & 7;
-            uint4 val = xv[u];
-            if (norm) {
-                const bf16 *he = reinterpret_cast<const bf16 *>(&xv[u]);
-                const bf16 *ge = reinterpret_cast<const bf16 *>(&gv[u]);
-                bf16 *oe = reinterpret_cast<bf16 *>(&val);
-                const float rs = s_rms[m];
-#pragma unroll
-                for (int e = 0; e < 8; ++e) oe[e] = f2bf(__fmul_rn(bf2f(ge[e]), rbf(__fmul_rn(bf2f(he[e]), rs))));
-            }
-            *reinterpret_cast<uint4 *>(sb + (size_t)atom * P.bn * 128 + m * 128 + ((cc ^ (m & 7)) << 4)) = val;
+        for (int e = 0; e < 4; ++e) {
+            const float2 f = __bfloat1622float2(v2[e]);
+            v2[e] = __hmul2(g2[e], __floats2bfloat162_rn(__fmul_rn(f.x, rs), __fmul_rn(f.y, rs)));
         }
+        *p = val;
     }
 }
 
@@ -466,163 +477,180 @@ __device__ __noinline__ void build_b_act(const MKParams &P, int slice, uint8_t *
     }
 }
 
-// q|k|v tile: adapter delta, bf16, per-head RMSNorm + RoPE for q and k, store q / paged K, V
+// q|k|v tile: adapter delta, bf16, per-head RMSNorm + RoPE for q and k, store q / paged K, V.
+// Lane l reduces the four consecutive features 4l..4l+3 of the 128-feature tile (one head of 128,
+// or two heads of 64: lanes 0-15 the first); the RoPE partner of feature i (i + DH/2 within the
+// head) sits in lane l ^ (DH/8).  Per pass row m: rowpos[m] its position (-1 beyond the RoPE
+// table), rowkv[m] its KV slot (page << 4 | slot in page; -1 beyond the reserved pages), both set
+// at kernel start.
 template <int DH, bool AD>
 __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, int cw, int lane, int m0, int mstep,
-                                       uint32_t tag, unsigned long long *st) {
-    constexpr int E = DH / 32;
+                                       uint32_t tag, const int *rowpos, const int *rowkv, unsigned long long *st) {
+    constexpr int LPH = DH / 4;  // lanes per head
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r;
-    const int heads_per_tile = TILE_ROWS / DH;
+    const int qw = dm.Hq * DH, kvw = dm.Hkv * DH, ft = tile * TILE_ROWS;
+    const int kind = ft < qw ? 0 : (ft < qw + kvw ? 1 : 2);
+    const int hl = lane / LPH, e0 = 4 * (lane % LPH);  // head within the tile, first element in the head
+    const int head = (ft - (kind == 0 ? 0 : (kind == 1 ? qw : qw + kvw))) / DH + hl;
+    const int f0 = ft + 4 * lane;
+    const bool lo = e0 < DH / 2;  // first half of the head (RoPE: x cos - partner sin)
     const bf16 *lb = P.lora_b[0] + (size_t)layer * P.lb_stride[0];
-    const int nrow = m0 < M ? (M - m0 + mstep - 1) / mstep : 0;
-    for (int it = cw; it < nrow * heads_per_tile; it += CT / 32) {
-        const int m = m0 + (it / heads_per_tile) * mstep, hh = it % heads_per_tile;
-        const int fbase = tile * TILE_ROWS + hh * DH;
-        const int qw = dm.Hq * DH, kvw = dm.Hkv * DH;
-        const int kind = fbase < qw ? 0 : (fbase < qw + kvw ? 1 : 2);
-        const int head = kind == 0 ? fbase / DH : (kind == 1 ? (fbase - qw) / DH : (fbase - qw - kvw) / DH);
-        const int b = P.pd.b0 + m / P.pd.R;
-        const int pos = P.L[b] + m % P.pd.R;
-        // features 0..E-1: the lane's outputs; feature E: the adapter row whose u lane j < r sums
-        int f[E + 1];
+    float g[4];
+    if (kind < 2) {
+        const uint2 graw = __ldg(reinterpret_cast<const uint2 *>((kind == 0 ? P.q_norm : P.k_norm) + (size_t)layer * DH + e0));
+        const float2 ga = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&graw.x));
+        const float2 gb = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&graw.y));
+        g[0] = ga.x, g[1] = ga.y, g[2] = gb.x, g[3] = gb.y;
+    }
+    BRow br[4];
+    if (AD)
 #pragma unroll
-        for (int j = 0; j < E; ++j) f[j] = fbase + lane + 32 * j;
-        f[E] = P.n_main[0] + kind * r + (lane < r ? lane : 0);
-        BRow br[E];  // the lane's B rows, in flight with the partial sums
-        if (AD)
-#pragma unroll
-            for (int j = 0; j < E; ++j) br[j] = load_brow(lb + (size_t)f[j] * r, r);
-        float y[E + 1];
-        sum_parts<E + (AD ? 1 : 0), AD ? 4 : 8>(P, 0, m, f, y, tag);
-        unsigned long long *sw = (it == 0 && lane == 0) ? st : nullptr;  // first row's sub-steps
+        for (int j = 0; j < 4; ++j) br[j] = load_brow(lb + (size_t)(f0 + j) * r, r);
+#pragma unroll 1
+    for (int m = m0 + cw * mstep; m < M; m += (CT / 32) * mstep) {
+        const int pos = rowpos[m];
+        // the RoPE factors go out before the partial sums and land while they poll
+        float4 cs4[2];
+        if (kind < 2 && pos >= 0) {
+            const float4 *c4 = reinterpret_cast<const float4 *>(P.rope_cs + (size_t)pos * (DH / 2) + (e0 % (DH / 2)));
+            cs4[0] = __ldg(c4);
+            cs4[1] = __ldg(c4 + 1);
+        }
+        float y[5];
+        sum_parts<2, AD, AD ? 4 : 8>(P, 0, m, f0, P.n_main[0] + kind * r + (lane < r ? lane : 0), y, tag);
+        unsigned long long *sw = (cw == 0 && m == m0 + cw * mstep && lane == 0) ? st : nullptr;  // first row
         stamp_at(sw, 9);
         float u[MAX_RANK];
-        if (AD) share_u(y[E], 0, u);
+        if (AD) share_u(y[4], 0, u);
 #pragma unroll
-        for (int j = 0; j < E; ++j) {
+        for (int j = 0; j < 4; ++j) {
             if (AD) y[j] = __fadd_rn(y[j], __fmul_rn(dm.lora_scale, lora_dot_w(u, br[j], r)));
             y[j] = rbf(y[j]);
         }
         if (kind < 2) {
-            const bf16 *gn = (kind == 0 ? P.q_norm : P.k_norm) + (size_t)layer * DH;
-            float ss = 0.f;
+            float ss = __fmul_rn(y[0], y[0]);
 #pragma unroll
-            for (int j = 0; j < E; ++j) ss = __fadd_rn(ss, __fmul_rn(y[j], y[j]));
+            for (int j = 1; j < 4; ++j) ss = __fadd_rn(ss, __fmul_rn(y[j], y[j]));
 #pragma unroll
-            for (int off = 16; off >= 1; off >>= 1) ss = __fadd_rn(ss, __shfl_xor_sync(0xffffffffu, ss, off));
-            ss = __shfl_sync(0xffffffffu, ss, 0);
+            for (int off = LPH / 2; off >= 1; off >>= 1) ss = __fadd_rn(ss, __shfl_xor_sync(0xffffffffu, ss, off));
             const float rs = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(__fdiv_rn(ss, (float)DH), dm.eps)));
 #pragma unroll
-            for (int j = 0; j < E; ++j) y[j] = rbf(__fmul_rn(bf2f(gn[lane + 32 * j]), rbf(__fmul_rn(y[j], rs))));
-            if (pos >= P.rope_rows) {
+            for (int j = 0; j < 4; ++j) y[j] = rbf(__fmul_rn(g[j], rbf(__fmul_rn(y[j], rs))));
+            const float *cs = reinterpret_cast<const float *>(cs4);  // cos, sin of elements e0..e0+3
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const float partner = __shfl_xor_sync(0xffffffffu, y[j], LPH / 2);
+                const float c = cs[2 * j], sn = cs[2 * j + 1];
+                y[j] = lo ? rbf(__fsub_rn(__fmul_rn(y[j], c), __fmul_rn(partner, sn)))
+                          : rbf(__fadd_rn(__fmul_rn(y[j], c), __fmul_rn(partner, sn)));
+            }
+            if (pos < 0) {
                 latch_error(P.status, DEV_BAD_POSITION);
                 continue;
-            }
-#pragma unroll
-            for (int j = 0; j < E / 2; ++j) {
-                const int e = lane + 32 * j;
-                const float2 cs = P.rope_cs[(size_t)pos * (DH / 2) + e];
-                const float a = y[j], c = y[j + E / 2];
-                y[j] = rbf(__fsub_rn(__fmul_rn(a, cs.x), __fmul_rn(c, cs.y)));
-                y[j + E / 2] = rbf(__fadd_rn(__fmul_rn(c, cs.x), __fmul_rn(a, cs.y)));
             }
         }
         stamp_at(sw, 10);
+        bf16 *dst;
         if (kind == 0) {
-            bf16 *dst = P.q + ((size_t)m * dm.Hq + head) * DH;
-#pragma unroll
-            for (int j = 0; j < E; ++j) dst[lane + 32 * j] = f2bf(y[j]);
+            dst = P.q + ((size_t)m * dm.Hq + head) * DH + e0;
         } else {
-            const int pg = pos / PAGE;
-            if (pg >= P.kv.pages_per_seq) {
+            const int rk = rowkv[m];
+            if (rk < 0) {
                 latch_error(P.status, DEV_BAD_POSITION);
                 continue;
             }
-            const int page = P.kv.page_table[b * P.kv.pages_per_seq + pg];
-            const size_t off = ((((size_t)layer * P.kv.n_pages + page) * dm.Hkv + head) * PAGE + (pos % PAGE)) * DH;
-            bf16 *dst = static_cast<bf16 *>(kind == 1 ? P.kv.k : P.kv.v) + off;
-#pragma unroll
-            for (int j = 0; j < E; ++j) dst[lane + 32 * j] = f2bf(y[j]);
+            dst = static_cast<bf16 *>(kind == 1 ? P.kv.k : P.kv.v) +
+                  ((((size_t)layer * P.kv.n_pages + (rk >> 4)) * dm.Hkv + head) * PAGE + (rk & 15)) * DH + e0;
         }
+        uint2 o;
+        *reinterpret_cast<__nv_bfloat162 *>(&o.x) = __floats2bfloat162_rn(y[0], y[1]);
+        *reinterpret_cast<__nv_bfloat162 *>(&o.y) = __floats2bfloat162_rn(y[2], y[3]);
+        *reinterpret_cast<uint2 *>(dst) = o;
         stamp_at(sw, 11);
     }
 }
 
-// o or down tile: adapter delta, residual add into h, per-tile sum of squares
+// o or down tile: adapter delta, residual add into h, per-tile sum of squares.  Lane l reduces the
+// four consecutive features 4l..4l+3 of the tile; the tile's sum of squares adds them in order,
+// then across the lanes by a fixed butterfly.
 template <bool AD>
 __device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int layer, int tile, int cw, int lane, int m0,
                                              int mstep, uint32_t tag, unsigned long long *st) {
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r, H = dm.H, nt = H / TILE_ROWS;
+    const int f0 = tile * TILE_ROWS + 4 * lane;
     const bf16 *lb = P.lora_b[lin] + (size_t)layer * P.lb_stride[lin];
-    if (m0 + cw * mstep >= M) return;
     // B rows depend only on the feature: loaded once, before the rows
     BRow br[4];
     if (AD)
 #pragma unroll
-        for (int e = 0; e < 4; ++e) br[e] = load_brow(lb + (size_t)(tile * TILE_ROWS + lane + 32 * e) * r, r);
+        for (int e = 0; e < 4; ++e) br[e] = load_brow(lb + (size_t)(f0 + e) * r, r);
+#pragma unroll 1
     for (int m = m0 + cw * mstep; m < M; m += (CT / 32) * mstep) {
-        // features 0-3: the lane's outputs; feature 4: the adapter row whose u lane j < r sums
-        int f[5];
-        float hv[4], acc[5];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            f[e] = tile * TILE_ROWS + lane + 32 * e;
-            hv[e] = bf2f(ldcg_bf(P.h + (size_t)m * H + f[e]));
-        }
-        f[4] = P.n_main[lin] + (lane < r ? lane : 0);
-        sum_parts<AD ? 5 : 4, AD ? 4 : 8>(P, lin, m, f, acc, tag);
+        uint2 *hp = reinterpret_cast<uint2 *>(P.h + (size_t)m * H + f0);
+        const uint2 hraw = __ldcg(hp);
+        float acc[5];
+        sum_parts<2, AD, AD ? 4 : 8>(P, lin, m, f0, P.n_main[lin] + (lane < r ? lane : 0), acc, tag);
         unsigned long long *sw = (cw == 0 && m == m0 && lane == 0) ? st : nullptr;  // first row's sub-steps
         stamp_at(sw, 9);
         float u[MAX_RANK];
         if (AD) share_u(acc[4], 0, u);
+        const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&hraw);
+        const float2 ha = __bfloat1622float2(h2[0]), hb = __bfloat1622float2(h2[1]);
+        const float hv[4] = {ha.x, ha.y, hb.x, hb.y};
         float v[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
             if (AD) acc[e] = __fadd_rn(acc[e], __fmul_rn(dm.lora_scale, lora_dot_w(u, br[e], r)));
             v[e] = rbf(__fadd_rn(hv[e], rbf(acc[e])));
-            P.h[(size_t)m * H + f[e]] = f2bf(v[e]);
         }
+        uint2 o;
+        *reinterpret_cast<__nv_bfloat162 *>(&o.x) = __floats2bfloat162_rn(v[0], v[1]);
+        *reinterpret_cast<__nv_bfloat162 *>(&o.y) = __floats2bfloat162_rn(v[2], v[3]);
+        *hp = o;
         stamp_at(sw, 10);
-        const float s = tile_sumsq(v);
-        if (lane == 0) P.ss[(size_t)m * nt + tile] = s;
+        float sq = __fmul_rn(v[0], v[0]);
+#pragma unroll
+        for (int e = 1; e < 4; ++e) sq = __fadd_rn(sq, __fmul_rn(v[e], v[e]));
+#pragma unroll
+        for (int off = 16; off >= 1; off >>= 1) sq = __fadd_rn(sq, __shfl_xor_sync(0xffffffffu, sq, off));
+        if (lane == 0) P.ss[(size_t)m * nt + tile] = sq;
         stamp_at(sw, 11);
     }
 }
 
-// gate|up tile (rows 0-63 gate features 64t.., rows 64-127 up features 64t..): SiLU(gate)*up
+// gate|up tile (rows 0-63 gate features 64t.., rows 64-127 up features 64t..): SiLU(gate)*up.
+// Lane l produces act features 64t + 2l and 64t + 2l + 1 (tile rows 2l, 2l + 1 and 64 + 2l,
+// 64 + 2l + 1) and stores them as one tagged word.
 template <bool AD>
 __device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, int cw, int lane, int m0, int mstep,
                                       uint32_t tag, unsigned long long *st) {
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r, I = dm.I;
+    const int a0 = tile * 64 + 2 * lane;  // the lane's first act feature
     const bf16 *lb = P.lora_b[2] + (size_t)layer * P.lb_stride[2];
-    if (m0 + cw * mstep >= M) return;
     BRow bg[2], bu[2];
     if (AD)
 #pragma unroll
         for (int e = 0; e < 2; ++e) {
-            const int a = tile * 64 + lane + 32 * e;
-            bg[e] = load_brow(lb + (size_t)a * r, r);
-            bu[e] = load_brow(lb + (size_t)(I + a) * r, r);
+            bg[e] = load_brow(lb + (size_t)(a0 + e) * r, r);
+            bu[e] = load_brow(lb + (size_t)(I + a0 + e) * r, r);
         }
+#pragma unroll 1
     for (int m = m0 + cw * mstep; m < M; m += (CT / 32) * mstep) {
-        // partial rows: gate j = lane, lane+32 at tile rows j; up at tile rows 64 + j; feature 4:
-        // adapter row lane (lanes 0..r-1 sum u_gate, lanes r..2r-1 u_up)
-        const int f[5] = {tile * TILE_ROWS + lane, tile * TILE_ROWS + lane + 32, tile * TILE_ROWS + 64 + lane,
-                          tile * TILE_ROWS + 96 + lane, P.n_main[2] + (lane < 2 * r ? lane : 0)};
+        // sums: gate pair, up pair; feature 4: adapter row lane (lanes 0..r-1 sum u_gate, r..2r-1 u_up)
         float ug[MAX_RANK], uu[MAX_RANK], s[5];
-        sum_parts<AD ? 5 : 4, 2>(P, 2, m, f, s, tag);
+        sum_parts<64, AD, 2>(P, 2, m, tile * TILE_ROWS + 2 * lane, P.n_main[2] + (lane < 2 * r ? lane : 0), s, tag);
         unsigned long long *sw = (cw == 0 && m == m0 && lane == 0) ? st : nullptr;  // first row's sub-steps
         stamp_at(sw, 9);
         if (AD) {
             share_u(s[4], 0, ug);
             share_u(s[4], r, uu);
         }
+        uint32_t bits[2];
 #pragma unroll
         for (int e = 0; e < 2; ++e) {
-            const int a = tile * 64 + lane + 32 * e;  // act feature
             float g = s[e], up = s[2 + e];
             if (AD) {
                 g = __fadd_rn(g, __fmul_rn(dm.lora_scale, lora_dot_w(ug, bg[e], r)));
@@ -631,12 +659,9 @@ __device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, i
             g = rbf(g);
             up = rbf(up);
             const float sg = __fdiv_rn(g, __fadd_rn(1.0f, expf(-g)));
-            // features a (even lane) and a + 1 (odd neighbour) go out as one tagged word
-            const uint32_t bits = __bfloat16_as_ushort(f2bf(__fmul_rn(sg, up)));
-            const uint32_t hi = __shfl_down_sync(0xffffffffu, bits, 1);
-            if ((lane & 1) == 0)
-                st_relaxed_u64(P.act + ((size_t)m * I + a) / 2, ((unsigned long long)tag << 32) | (hi << 16) | bits);
+            bits[e] = __bfloat16_as_ushort(f2bf(__fmul_rn(sg, up)));
         }
+        st_relaxed_u64(P.act + ((size_t)m * I + a0) / 2, ((unsigned long long)tag << 32) | (bits[1] << 16) | bits[0]);
         stamp_at(sw, 11);
     }
 }
@@ -652,25 +677,43 @@ __device__ __forceinline__ uint32_t sw128(int row, int colb) {
     return (uint32_t)(row * 128 + ((((colb >> 4) ^ (row & 7)) << 4) | (colb & 15)));
 }
 
-// TMA loads of the pages of one attention split (thread 0 of the compute group).
+// TMA loads of the pages of one attention split, issued by one thread of the compute group.
 // stage 0: pages entirely below the cached length L (written by earlier passes: prefetched
-// before the item's inputs are ready); stage 1: pages holding this pass's block rows.
-// Returns the bytes of the chosen pages; issues the copies only when `issue` is set.
-__device__ uint32_t attn_pages(const MKParams &P, int layer, int bl, int g, int s, int stage, uint8_t *smem,
-                               uint64_t *bar, bool issue) {
+// before the item's inputs are ready); stage 1: pages holding this pass's block rows.  Announces
+// the stage's bytes on `bar` (stage 1 with the item's one arrival) before issuing the copies.
+// The page-table entries are read together first (one round trip), kept in `phys` (8 shared ints
+// owned by the calling thread).  Returns the stage's bytes.
+__device__ __noinline__ uint32_t attn_pages(const MKParams &P, int layer, int bl, int g, int s, int stage,
+                                            uint8_t *smem, uint64_t *bar, int *phys) {
+    constexpr int NP = ATT_SPLIT / PAGE;
     const int b = P.pd.b0 + bl;
-    const int L = P.L[b], T = L + P.pd.R, k0 = s * ATT_SPLIT;
-    const int subs = P.dm.d / 64;
-    uint32_t bytes = 0;
-    for (int p = 0; p < ATT_SPLIT / PAGE; ++p) {
+    const int L = P.L[b], T = L + P.pd.R, k0 = s * ATT_SPLIT, pg0 = k0 / PAGE;
+    const int *pt = P.kv.page_table + (size_t)b * P.kv.pages_per_seq + pg0;
+    unsigned mask = 0;
+    int ph[NP];
+#pragma unroll
+    for (int p = 0; p < NP; ++p) {
         const int kp0 = k0 + p * PAGE;
-        if (kp0 >= T || kp0 / PAGE >= P.kv.pages_per_seq) continue;
-        const bool cached = kp0 + PAGE <= L;
-        if (cached != (stage == 0)) continue;
-        bytes += (uint32_t)subs * 2u * PAGE * 128u;
-        if (!issue) continue;
-        const int phys = P.kv.page_table[b * P.kv.pages_per_seq + kp0 / PAGE];
-        const int row0 = ((layer * P.kv.n_pages + phys) * P.dm.Hkv + g) * PAGE;
+        const bool ok = kp0 < T && pg0 + p < P.kv.pages_per_seq && ((kp0 + PAGE <= L) == (stage == 0));
+        mask |= (ok ? 1u : 0u) << p;
+        ph[p] = ok ? pt[p] : 0;
+    }
+#pragma unroll
+    for (int p = 0; p < NP; ++p) phys[p] = ph[p];
+    const int subs = P.dm.d / 64;
+    const uint32_t bytes = (uint32_t)__popc(mask) * (uint32_t)subs * 2u * PAGE * 128u;
+    // the block's pages were written by this pass's q|k|v reducers (generic stores, acquired
+    // before this call): order them before the TMA reads
+    if (stage == 1 && mask) fence_proxy_async_global();
+    if (stage == 1)
+        mbar_arrive_expect_tx(bar, bytes);
+    else if (bytes)
+        mbar_expect_tx(bar, bytes);
+#pragma unroll 1
+    for (int p = 0; p < NP; ++p) {
+        if (!((mask >> p) & 1u)) continue;
+        const int row0 = ((layer * P.kv.n_pages + phys[p]) * P.dm.Hkv + g) * PAGE;
+#pragma unroll 1
         for (int sub = 0; sub < subs; ++sub) {
             tma_load_2d(smem + sub * ATT_SUB_BYTES + p * PAGE * 128, &P.kmap, sub * 64, row0, bar);
             tma_load_2d(smem + (subs + sub) * ATT_SUB_BYTES + p * PAGE * 128, &P.vmap, sub * 64, row0, bar);
@@ -680,14 +723,17 @@ __device__ uint32_t attn_pages(const MKParams &P, int layer, int bl, int g, int 
 }
 
 // One (sequence, KV head, 128-key split) on the compute group, after its K/V pages landed in
-// `smem` (stages 0 and 1 of attn_pages) and `bar` completed phase `parity`.
+// `smem` (stages 0 and 1 of attn_pages) and `bar` completed phase `parity`.  Each warp takes one
+// 16-row query tile and one 64-key half of the split; the halves are separate partial results
+// (m, l, O) that the merge combines like splits.  Within a half the keys go in chunks of 16 with
+// a running maximum (online softmax): scores by bf16 mma.sync, the row maximum and the weights in
+// fp32, P (weights) in fp16 against V converted to fp16, O in fp32.  The loop over chunks is not
+// unrolled: the code stays small enough for the instruction cache.
 template <int DH, bool BLK>
 __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, int g, int s, uint8_t *smem,
                                         uint64_t *bar, uint32_t parity, int ct, int cw, int lane,
                                         unsigned long long *stamp) {
-    // each warp takes one 16-row query tile and one half of the split's keys; the halves are
-    // separate partial results (m, l, O) that the merge combines like splits
-    constexpr int NT = ATT_SPLIT / 8 / ATT_SUBS, KS = DH / 16, DT = DH / 8, SUBS = DH / 64;
+    constexpr int KS = DH / 16, DT = DH / 8, SUBS = DH / 64;
     constexpr int HALF = ATT_SPLIT / ATT_SUBS;
     const Dims &dm = P.dm;
     const int b = P.pd.b0 + bl;
@@ -701,156 +747,162 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
     uint8_t *sK = smem, *sV = smem + SUBS * ATT_SUB_BYTES;
     // pages without keys of this pass were not loaded: zero their V rows (p = 0 there, and
     // 0 * stale bits could be NaN); their K rows are masked
-    for (int idx = ct; idx < (ATT_SPLIT / PAGE) * PAGE * SUBS * 8; idx += CT) {
-        const int chunk = idx % 8, row = (idx / 8) % ATT_SPLIT, sub = idx / (8 * ATT_SPLIT);
-        const int kp0 = k0 + (row / PAGE) * PAGE;
-        if (kp0 >= T || kp0 / PAGE >= P.kv.pages_per_seq)
-            *reinterpret_cast<uint4 *>(sV + sub * ATT_SUB_BYTES + row * 128 + chunk * 16) = make_uint4(0, 0, 0, 0);
+    const int kv_end = min(T, P.kv.pages_per_seq * PAGE);  // keys at or past this were not loaded
+    if (k0 + ATT_SPLIT > kv_end) {
+        const int row0 = max(0, (kv_end - k0 + PAGE - 1) / PAGE * PAGE);
+#pragma unroll 1
+        for (int idx = row0 * 8 * SUBS + ct; idx < ATT_SPLIT * 8 * SUBS; idx += CT) {
+            const int sub = idx & (SUBS - 1), rc = idx / SUBS;  // (row, chunk) = rc / 8, rc % 8
+            *reinterpret_cast<uint4 *>(sV + sub * ATT_SUB_BYTES + (rc >> 3) * 128 + (rc & 7) * 16) = make_uint4(0, 0, 0, 0);
+        }
     }
     const bool landed = mbar_wait_mk(bar, parity, P, DEV_TIMEOUT_LOAD);
     if (stamp && ct == 0) stamp[4] = globaltimer_ns();
     // V to fp16 in place (each 16-byte chunk independently; the swizzle layout is unchanged)
+#pragma unroll 1
     for (int idx = ct; idx < SUBS * ATT_SUB_BYTES / 16; idx += CT) {
         uint4 *p4 = reinterpret_cast<uint4 *>(sV + idx * 16);
-        const uint4 v4 = *p4;
-        const bf16 *ve = reinterpret_cast<const bf16 *>(&v4);
-        uint4 h4;
-        uint32_t *hw = reinterpret_cast<uint32_t *>(&h4);
+        uint4 v4 = *p4;
+        uint32_t *w = reinterpret_cast<uint32_t *>(&v4);
 #pragma unroll
-        for (int e = 0; e < 4; ++e) hw[e] = pack_half2(bf2f(ve[2 * e]), bf2f(ve[2 * e + 1]));
-        *p4 = h4;
+        for (int e = 0; e < 4; ++e) {
+            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[e]));
+            w[e] = pack_half2(f.x, f.y);
+        }
+        *p4 = v4;
     }
     bar_compute();
     if (stamp && ct == 0) stamp[5] = globaltimer_ns();
     if (!landed) return;
     const int gq = lane >> 2, tq = lane & 3;
-    constexpr bool blk = BLK;  // draft mask: the block's mask rows see each other
+    const float scale = P.att_scale;
+#pragma unroll 1
     for (int unit = cw; unit < n_mt * ATT_SUBS; unit += CT / 32) {
         const int mt = unit / ATT_SUBS, half = unit % ATT_SUBS, kb = half * HALF;
         const int qv0 = mt * 16 + gq, qv1 = qv0 + 8;
         const bool val0 = qv0 < QV, val1 = qv1 < QV;
         const int i0 = val0 ? qv0 / grp : 0, i1 = val1 ? qv1 / grp : 0;
         const int h0 = g * grp + (val0 ? qv0 % grp : 0), h1 = g * grp + (val1 ? qv1 % grp : 0);
-        const bf16 *q0 = P.q + ((size_t)(bl * R + i0) * dm.Hq + h0) * DH;
-        const bf16 *q1 = P.q + ((size_t)(bl * R + i1) * dm.Hq + h1) * DH;
-        uint32_t qa[KS][4];
-#pragma unroll
-        for (int ks = 0; ks < KS; ++ks) {
-            const int c = ks * 16 + 2 * tq;
-            qa[ks][0] = val0 ? __ldcg(reinterpret_cast<const unsigned *>(q0 + c)) : 0u;
-            qa[ks][1] = val1 ? __ldcg(reinterpret_cast<const unsigned *>(q1 + c)) : 0u;
-            qa[ks][2] = val0 ? __ldcg(reinterpret_cast<const unsigned *>(q0 + c + 8)) : 0u;
-            qa[ks][3] = val1 ? __ldcg(reinterpret_cast<const unsigned *>(q1 + c + 8)) : 0u;
-        }
         unsigned long long *sw = (unit == 0 && lane == 0) ? stamp : nullptr;  // first unit's sub-steps
-        float sc[NT][4];
+        uint32_t qa[KS][4];
+        {
+            const bf16 *q0 = P.q + ((size_t)(bl * R + i0) * dm.Hq + h0) * DH + 2 * tq;
+            const bf16 *q1 = P.q + ((size_t)(bl * R + i1) * dm.Hq + h1) * DH + 2 * tq;
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-            sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
-            // K fragments of two k-steps per ldmatrix.x4: matrix j = keys n0..n0+7, dims 8j..8j+7
-            // of the 32-dim chunk; thread t addresses row t % 8 of matrix t / 8
-            const int kr = kb + nt * 8 + (lane & 7);
-#pragma unroll
-            for (int ks = 0; ks < KS; ks += 2) {
-                const int e = ks * 16 + (lane >> 3) * 8;
-                const uint32_t addr = smem_u32(sK + (e >> 6) * ATT_SUB_BYTES + sw128(kr, (e & 63) * 2));
-                uint32_t b0, b1, b2, b3;
-                asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
-                             : "=r"(b0), "=r"(b1), "=r"(b2), "=r"(b3)
-                             : "r"(addr));
-                mma_m16n8k16_bf16(sc[nt], qa[ks], b0, b1);
-                mma_m16n8k16_bf16(sc[nt], qa[ks + 1], b2, b3);
+            for (int ks = 0; ks < KS; ++ks) {
+                qa[ks][0] = val0 ? __ldcg(reinterpret_cast<const unsigned *>(q0 + ks * 16)) : 0u;
+                qa[ks][1] = val1 ? __ldcg(reinterpret_cast<const unsigned *>(q1 + ks * 16)) : 0u;
+                qa[ks][2] = val0 ? __ldcg(reinterpret_cast<const unsigned *>(q0 + ks * 16 + 8)) : 0u;
+                qa[ks][3] = val1 ? __ldcg(reinterpret_cast<const unsigned *>(q1 + ks * 16 + 8)) : 0u;
             }
         }
-        stamp_at(sw, 9);
-        const int qp0 = L + i0, qp1 = L + i1;
         // last visible key of each row: causal rows see up to themselves; in the draft the
         // block's mask rows (i >= 1) also see the rest of the block
-        const int lim0 = val0 ? ((blk && i0 >= 1) ? T - 1 : qp0) : -1;
-        const int lim1 = val1 ? ((blk && i1 >= 1) ? T - 1 : qp1) : -1;
-        const float scale = P.att_scale;
-        float m0 = -INFINITY, m1 = -INFINITY;
+        const int lim0 = val0 ? ((BLK && i0 >= 1) ? T - 1 : L + i0) : -1;
+        const int lim1 = val1 ? ((BLK && i1 >= 1) ? T - 1 : L + i1) : -1;
+        float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+        float oc[DT][4];
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
+        for (int dt = 0; dt < DT; ++dt) oc[dt][0] = oc[dt][1] = oc[dt][2] = oc[dt][3] = 0.f;
+        const int kend = min(HALF, T - (k0 + kb));  // keys of the half that exist
+#pragma unroll 1
+        for (int c0 = 0; c0 < kend; c0 += 16) {
+            float sc[2][4];
 #pragma unroll
-            for (int e = 0; e < 2; ++e) {
-                const int kp = k0 + kb + nt * 8 + 2 * tq + e;
-                const bool vis0 = kp <= lim0;
-                const bool vis1 = kp <= lim1;
-                sc[nt][e] = vis0 ? __fmul_rn(sc[nt][e], scale) : -INFINITY;
-                sc[nt][2 + e] = vis1 ? __fmul_rn(sc[nt][2 + e], scale) : -INFINITY;
-                m0 = fmaxf(m0, sc[nt][e]);
-                m1 = fmaxf(m1, sc[nt][2 + e]);
+            for (int nt = 0; nt < 2; ++nt) {
+                sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
+                // K fragments of two k-steps per ldmatrix.x4: matrix j = keys n0..n0+7, dims 8j..8j+7
+                // of the 32-dim chunk; thread t addresses row t % 8 of matrix t / 8
+                const int kr = kb + c0 + nt * 8 + (lane & 7);
+#pragma unroll
+                for (int ks = 0; ks < KS; ks += 2) {
+                    const int e = ks * 16 + (lane >> 3) * 8;
+                    const uint32_t addr = smem_u32(sK + (e >> 6) * ATT_SUB_BYTES + sw128(kr, (e & 63) * 2));
+                    uint32_t b0, b1, b2, b3;
+                    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                                 : "=r"(b0), "=r"(b1), "=r"(b2), "=r"(b3)
+                                 : "r"(addr));
+                    mma_m16n8k16_bf16(sc[nt], qa[ks], b0, b1);
+                    mma_m16n8k16_bf16(sc[nt], qa[ks + 1], b2, b3);
+                }
+            }
+            float c0m = -INFINITY, c1m = -INFINITY;
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const int kp = k0 + kb + c0 + nt * 8 + 2 * tq + e;
+                    sc[nt][e] = kp <= lim0 ? __fmul_rn(sc[nt][e], scale) : -INFINITY;
+                    sc[nt][2 + e] = kp <= lim1 ? __fmul_rn(sc[nt][2 + e], scale) : -INFINITY;
+                    c0m = fmaxf(c0m, sc[nt][e]);
+                    c1m = fmaxf(c1m, sc[nt][2 + e]);
+                }
+            c0m = fmaxf(c0m, __shfl_xor_sync(0xffffffffu, c0m, 1));
+            c0m = fmaxf(c0m, __shfl_xor_sync(0xffffffffu, c0m, 2));
+            c1m = fmaxf(c1m, __shfl_xor_sync(0xffffffffu, c1m, 1));
+            c1m = fmaxf(c1m, __shfl_xor_sync(0xffffffffu, c1m, 2));
+            const float n0 = fmaxf(m0, c0m), n1 = fmaxf(m1, c1m);
+            // rescale what was summed so far to the new maximum (nothing was, while it is -inf)
+            const float a0 = m0 == -INFINITY ? 0.f : __expf(m0 - n0), a1 = m1 == -INFINITY ? 0.f : __expf(m1 - n1);
+            const float z0 = n0 == -INFINITY ? 0.f : n0, z1 = n1 == -INFINITY ? 0.f : n1;
+            m0 = n0;
+            m1 = n1;
+            l0 = __fmul_rn(l0, a0);
+            l1 = __fmul_rn(l1, a1);
+#pragma unroll
+            for (int dt = 0; dt < DT; ++dt) {
+                oc[dt][0] = __fmul_rn(oc[dt][0], a0);
+                oc[dt][1] = __fmul_rn(oc[dt][1], a0);
+                oc[dt][2] = __fmul_rn(oc[dt][2], a1);
+                oc[dt][3] = __fmul_rn(oc[dt][3], a1);
+            }
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    sc[nt][e] = sc[nt][e] == -INFINITY ? 0.f : __expf(sc[nt][e] - z0);
+                    sc[nt][2 + e] = sc[nt][2 + e] == -INFINITY ? 0.f : __expf(sc[nt][2 + e] - z1);
+                    l0 += sc[nt][e];
+                    l1 += sc[nt][2 + e];
+                }
+            // P as the fp16 A fragment of one 16-key step
+            uint32_t pa[4];
+            pa[0] = pack_half2(sc[0][0], sc[0][1]);
+            pa[1] = pack_half2(sc[0][2], sc[0][3]);
+            pa[2] = pack_half2(sc[1][0], sc[1][1]);
+            pa[3] = pack_half2(sc[1][2], sc[1][3]);
+            const int vrow = kb + c0 + (lane & 7) + ((lane >> 3) & 1) * 8;
+#pragma unroll
+            for (int dt = 0; dt < DT; dt += 2) {
+                const int vcol = dt * 8 + (lane >> 4) * 8;
+                const uint32_t addr = smem_u32(sV + (vcol >> 6) * ATT_SUB_BYTES + sw128(vrow, (vcol & 63) * 2));
+                uint32_t r0, r1, r2, r3;
+                asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                             : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                             : "r"(addr));
+                mma_m16n8k16_f16(oc[dt], pa, r0, r1);
+                mma_m16n8k16_f16(oc[dt + 1], pa, r2, r3);
             }
         }
-        m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, 1));
-        m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, 2));
-        m1 = fmaxf(m1, __shfl_xor_sync(0xffffffffu, m1, 1));
-        m1 = fmaxf(m1, __shfl_xor_sync(0xffffffffu, m1, 2));
-        const float mz0 = m0 == -INFINITY ? 0.f : m0, mz1 = m1 == -INFINITY ? 0.f : m1;
-        float l0 = 0.f, l1 = 0.f;
-#pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-                const float p0 = sc[nt][e] == -INFINITY ? 0.f : __expf(sc[nt][e] - mz0);
-                const float p1 = sc[nt][2 + e] == -INFINITY ? 0.f : __expf(sc[nt][2 + e] - mz1);
-                sc[nt][e] = p0;
-                sc[nt][2 + e] = p1;
-                l0 += p0;
-                l1 += p1;
-            }
-        }
+        stamp_at(sw, 10);
         l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
         l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
         l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
         l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-        // P as fp16 A fragments (k-step = 16 keys); the fp32 scores are dead from here on
-        uint32_t pa[HALF / 16][4];
-#pragma unroll
-        for (int kstep = 0; kstep < HALF / 16; ++kstep) {
-            pa[kstep][0] = pack_half2(sc[2 * kstep][0], sc[2 * kstep][1]);
-            pa[kstep][1] = pack_half2(sc[2 * kstep][2], sc[2 * kstep][3]);
-            pa[kstep][2] = pack_half2(sc[2 * kstep + 1][0], sc[2 * kstep + 1][1]);
-            pa[kstep][3] = pack_half2(sc[2 * kstep + 1][2], sc[2 * kstep + 1][3]);
-        }
-        stamp_at(sw, 10);
         const int nsa = P.att_splits_alloc;
         const int sub = s * ATT_SUBS + half;  // index of this partial result
-        float *dst0 = val0 ? P.o_part + (((size_t)(bl * R + i0) * dm.Hq + h0) * nsa + sub) * DH : nullptr;
-        float *dst1 = val1 ? P.o_part + (((size_t)(bl * R + i1) * dm.Hq + h1) * nsa + sub) * DH : nullptr;
-        // O = P V in halves of the head dimension (keeps the accumulators at 32 registers)
+        if (val0) {
+            float *dst = P.o_part + (((size_t)(bl * R + i0) * dm.Hq + h0) * nsa + sub) * DH + 2 * tq;
 #pragma unroll
-        for (int half = 0; half < 2; ++half) {
-            float oc[DT / 2][4];
-#pragma unroll
-            for (int dt = 0; dt < DT / 2; ++dt) oc[dt][0] = oc[dt][1] = oc[dt][2] = oc[dt][3] = 0.f;
-#pragma unroll
-            for (int kstep = 0; kstep < HALF / 16; ++kstep) {
-                const int vrow = kb + kstep * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-#pragma unroll
-                for (int dt = 0; dt < DT / 2; dt += 2) {
-                    const int vcol = (half * (DT / 2) + dt) * 8 + (lane >> 4) * 8;
-                    const uint32_t addr = smem_u32(sV + (vcol >> 6) * ATT_SUB_BYTES + sw128(vrow, (vcol & 63) * 2));
-                    uint32_t r0, r1, r2, r3;
-                    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-                                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-                                 : "r"(addr));
-                    mma_m16n8k16_f16(oc[dt], pa[kstep], r0, r1);
-                    mma_m16n8k16_f16(oc[dt + 1], pa[kstep], r2, r3);
-                }
-            }
-#pragma unroll
-            for (int dt = 0; dt < DT / 2; ++dt) {
-                const int col = (half * (DT / 2) + dt) * 8 + 2 * tq;
-                if (val0) *reinterpret_cast<float2 *>(dst0 + col) = make_float2(oc[dt][0], oc[dt][1]);
-                if (val1) *reinterpret_cast<float2 *>(dst1 + col) = make_float2(oc[dt][2], oc[dt][3]);
-            }
+            for (int dt = 0; dt < DT; ++dt) *reinterpret_cast<float2 *>(dst + dt * 8) = make_float2(oc[dt][0], oc[dt][1]);
+            if (tq == 0) P.ml_part[((size_t)(bl * R + i0) * dm.Hq + h0) * nsa + sub] = make_float2(m0, l0);
         }
-        if (val0 && tq == 0)
-            P.ml_part[((size_t)(bl * R + i0) * dm.Hq + h0) * nsa + sub] = make_float2(m0, l0);
-        if (val1 && tq == 0)
-            P.ml_part[((size_t)(bl * R + i1) * dm.Hq + h1) * nsa + sub] = make_float2(m1, l1);
+        if (val1) {
+            float *dst = P.o_part + (((size_t)(bl * R + i1) * dm.Hq + h1) * nsa + sub) * DH + 2 * tq;
+#pragma unroll
+            for (int dt = 0; dt < DT; ++dt) *reinterpret_cast<float2 *>(dst + dt * 8) = make_float2(oc[dt][2], oc[dt][3]);
+            if (tq == 0) P.ml_part[((size_t)(bl * R + i1) * dm.Hq + h1) * nsa + sub] = make_float2(m1, l1);
+        }
         stamp_at(sw, 11);
     }
 }
@@ -924,66 +976,18 @@ __device__ __noinline__ void attn_combine(const MKParams &P, int bl, int g, int 
 }
 
 // Attention merge mode of a (sequence, head) with nsp splits: shared by all splits when they sit
-// on distinct CTAs (nsp <= grid), else done by the last split; and the count that marks it done.
+// on distinct CTAs (nsp <= grid), else done by the last split.
 __device__ __forceinline__ bool att_shared_merge(int nsp) { return nsp <= (int)gridDim.x; }
-__device__ __forceinline__ int att_done(int nsp) { return att_shared_merge(nsp) ? 2 * nsp : nsp + 1; }
-
-// 128-row tiles that overlap features [f0, f1)
-__device__ __forceinline__ int tiles_over(int f0, int f1) { return (f1 - 1) / TILE_ROWS - f0 / TILE_ROWS + 1; }
-
-// KV head groups whose q, k or v features overlap q|k|v tile t: [*g0, *g1]
-__device__ __forceinline__ void qkv_tile_groups(const Dims &dm, int t, int *g0, int *g1) {
-    const int grp = dm.Hq / dm.Hkv, qw = dm.Hq * dm.d, kvw = dm.Hkv * dm.d;
-    const int f0 = t * TILE_ROWS, f1 = f0 + TILE_ROWS - 1;  // the tile lies in one of q, k, v
-    if (f0 < qw) {
-        *g0 = f0 / dm.d / grp;
-        *g1 = f1 / dm.d / grp;
-    } else {
-        const int base = f0 < qw + kvw ? qw : qw + kvw;
-        *g0 = (f0 - base) / dm.d;
-        *g1 = (f1 - base) / dm.d;
-    }
-}
-
-// slices stored by the reducers an attention item of group g waits for: every slice of every
-// q, k and v tile that holds a feature of the group
-__device__ __forceinline__ int att_in_target(const MKParams &P, int g) {
-    const Dims &dm = P.dm;
-    const int grp = dm.Hq / dm.Hkv, d = dm.d, qw = dm.Hq * d, kvw = dm.Hkv * d;
-    return P.ks[0] * (tiles_over(g * grp * d, (g + 1) * grp * d) + tiles_over(qw + g * d, qw + (g + 1) * d) +
-                      tiles_over(qw + kvw + g * d, qw + kvw + (g + 1) * d));
-}
 
 // the item's inputs are complete (one thread; false on abort)
-__device__ bool wait_deps(const MKParams &P, const MKItem &it) {
-    const Dims &dm = P.dm;
-    const int l = it.layer;
-    if (it.op == MK_LINEAR) {
-        const int s = it.b;
-        switch (it.lin) {
-            case 0:
-                if (l == 0) return spin_until(P.cnt + P.cl.embed, P.pd.M, P);
-                return spin_until(ctr(P, l - 1, P.cl.res_dn), dm.H / TILE_ROWS * P.ks[3], P);
-            case 1: {
-                const int w = P.katoms[1] * KT;
-                const int h0 = (s * w) / dm.d, h1 = (s * w + w - 1) / dm.d;
-                const int grp = dm.Hq / dm.Hkv;
-                for (int bl = 0; bl < P.pd.nb; ++bl)
-                    for (int g = h0 / grp; g <= h1 / grp; ++g)
-                        if (!spin_until(ctr(P, l, P.cl.att + bl * dm.Hkv + g), att_done(P.nsplit[bl]), P))
-                            return false;
-                return true;
-            }
-            case 2: return spin_until(ctr(P, l, P.cl.res_o), dm.H / TILE_ROWS * P.ks[1], P);
-            default:
-                // act words carry the tag of the gate|up reduction that wrote them: the operand
-                // staging polls them itself
-                return true;
-        }
-    }
-    if (it.op == MK_ATTN) return spin_until(ctr(P, l, P.cl.att_in + it.b), att_in_target(P, it.b), P);
-    if (it.op == MK_FINAL) return spin_until(ctr(P, P.pd.nl_run - 1, P.cl.res_dn), dm.H / TILE_ROWS * P.ks[3], P);
-    return true;
+__device__ __forceinline__ bool wait_deps(const MKParams &P, const MKItem &it) {
+    return it.wait_off < 0 || spin_until(P.cnt + it.wait_off, it.wait_tgt, P);
+}
+
+// one thread: the item's result is stored (and made visible to it by a barrier): count it
+__device__ __forceinline__ void release_item(const MKParams &P, const MKItem &it) {
+    if (it.rel[0] >= 0) red_release_add(P.cnt + it.rel[0], 1);
+    if (it.rel[1] >= 0) red_release_add(P.cnt + it.rel[1], 1);
 }
 
 // ------------------------------------------------------------------ the kernel
@@ -1003,6 +1007,10 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
     __shared__ int s_flag, s_red, s_ok;
     __shared__ uint32_t s_tag;  // this pass's partial-sum tag
     __shared__ float s_rms[MAX_ROWS];
+    __shared__ int s_phys[2][ATT_SPLIT / PAGE];  // page ids of attention stages 0 and 1
+    // per pass row: position (-1 beyond the RoPE table) and KV slot (page << 4 | slot; -1 beyond
+    // the reserved pages)
+    __shared__ int s_rowpos[MAX_ROWS], s_rowkv[MAX_ROWS];
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const MKItem *my = P.items + P.cta_off[blockIdx.x];
@@ -1029,6 +1037,11 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
         fence_mbarrier_init();
     }
     if (warp == 0) tmem_alloc(&tmem_slot, P.tmem_cols);
+    for (int m = tid; m < P.pd.M; m += MK_THREADS) {
+        const int b = P.pd.b0 + m / P.pd.R, pos = P.L[b] + m % P.pd.R, pg = pos / PAGE;
+        s_rowpos[m] = pos < P.rope_rows ? pos : -1;
+        s_rowkv[m] = pg < P.kv.pages_per_seq ? (P.kv.page_table[b * P.kv.pages_per_seq + pg] << 4) | (pos % PAGE) : -1;
+    }
     // zero the padding rows of the activation tile once (rows >= M are never written)
     for (int q = tid; q < (P.b_dbl ? MAX_ATOMS : HALF_ATOMS) * P.bn * 8; q += MK_THREADS) {
         const int atom = q / (P.bn * 8), rem = q % (P.bn * 8), m = rem / 8;
@@ -1137,8 +1150,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
             if (att_active && ct == CT_PAGES) {
                 // pages below the cached length do not depend on this pass: fetch them now (the
                 // barrier after the input wait orders this before the split's arrival)
-                mbar_expect_tx(&att_bar, attn_pages(P, it.layer, it.a, it.b, it.c, 0, uni, &att_bar, false));
-                attn_pages(P, it.layer, it.a, it.b, it.c, 0, uni, &att_bar, true);
+                attn_pages(P, it.layer, it.a, it.b, it.c, 0, uni, &att_bar, s_phys[0]);
                 att_pend = true;
             }
             if (ct == 0) s_flag = wait_deps(P, it) ? 1 : 0;
@@ -1148,7 +1160,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
             if (it.op == MK_EMBED) {
                 do_embed(P, it.a, cw, lane);
                 bar_compute();
-                if (ct == 0) red_release_add(P.cnt + P.cl.embed, 1);
+                if (ct == 0) release_item(P, it);
             } else if (it.op == MK_FINAL) {
                 const int r = it.a, m = it.b;
                 if (ct == 0) s_rms[0] = row_rms(P, m);
@@ -1169,12 +1181,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 const int bl = it.a, g = it.b, s = it.c;
                 if (att_active) {
                     if (ct == 0) {
-                        const uint32_t nb1 = attn_pages(P, it.layer, bl, g, s, 1, uni, &att_bar, false);
-                        // the block's pages were written by this pass's q|k|v reducers (generic
-                        // stores, acquired above); order them before the TMA reads
-                        if (nb1) fence_proxy_async_global();
-                        mbar_arrive_expect_tx(&att_bar, nb1);
-                        if (nb1) attn_pages(P, it.layer, bl, g, s, 1, uni, &att_bar, true);
+                        attn_pages(P, it.layer, bl, g, s, 1, uni, &att_bar, s_phys[1]);
                         if (tr) tr[MK_STAMPS * i + 8] = globaltimer_ns();
                     }
                     unsigned long long *st = tr ? tr + MK_STAMPS * i : nullptr;
@@ -1206,7 +1213,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                     const int p0 = shared_merge ? s : 0, pstep = shared_merge ? nsp : 1;
                     attn_combine<DH>(P, bl, g, cw, lane, p0, pstep, tr ? tr + MK_STAMPS * i : nullptr);
                     bar_compute();
-                    if (ct == 0) red_release_add(c, 1);
+                    if (ct == 0) release_item(P, it);  // counts on the o slice that reads the group
                     if (tr && ct == 0) tr[MK_STAMPS * i + 7] = globaltimer_ns();
                 }
             } else {
@@ -1218,24 +1225,24 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                     if (lin == 3)
                         build_b_act(P, s, uni, ct, s_tag + l, st_i);
                     else
-                        build_b(P, lin, l, s, uni, s_rms, ct, 0, na, true, st_i);
+                        build_b(P, lin, l, s, uni, s_rms, ct, 0, true, st_i);
                     fence_proxy_async();
                     bar_compute();
                     if (ct == 0) mbarrier_arrive_one(&b_full[0]);
                 } else if (P.b_dbl) {
                     // wide slice, both halves fit: the first half's MMAs run while the second is staged
-                    build_b(P, lin, l, s, uni, s_rms, ct, 0, HALF_ATOMS, true, st_i);
+                    build_b(P, lin, l, s, uni, s_rms, ct, 0, true, st_i);
                     fence_proxy_async();
                     bar_compute();
                     if (ct == 0) mbarrier_arrive_one(&b_full[0]);
-                    build_b(P, lin, l, s, uni + (size_t)HALF_ATOMS * P.bn * 128, s_rms, ct, HALF_ATOMS,
-                            na - HALF_ATOMS, false, nullptr);
+                    build_b(P, lin, l, s, uni + (size_t)HALF_ATOMS * P.bn * 128, s_rms, ct, HALF_ATOMS, false,
+                            nullptr);
                     fence_proxy_async();
                     bar_compute();
                     if (ct == 0) mbarrier_arrive_one(&b_full[1]);
                 } else {
                     // operand in two rounds through the same area
-                    build_b(P, lin, l, s, uni, s_rms, ct, 0, HALF_ATOMS, true, st_i);
+                    build_b(P, lin, l, s, uni, s_rms, ct, 0, true, st_i);
                     fence_proxy_async();
                     bar_compute();
                     if (ct == 0) {
@@ -1244,7 +1251,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                     }
                     bar_compute();
                     if (!s_ok) break;
-                    build_b(P, lin, l, s, uni, s_rms, ct, HALF_ATOMS, na - HALF_ATOMS, false, nullptr);
+                    build_b(P, lin, l, s, uni, s_rms, ct, HALF_ATOMS, false, nullptr);
                     fence_proxy_async();
                     bar_compute();
                     if (ct == 0) mbarrier_arrive_one(&b_full[1]);
@@ -1293,22 +1300,14 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
                 }
                 const uint32_t tag = s_tag + l;
                 if (lin == 0) {
-                    reduce_qkv<DH, DRAFT>(P, l, t, cw, lane, s, ks, tag, st_i);
+                    reduce_qkv<DH, DRAFT>(P, l, t, cw, lane, s, ks, tag, s_rowpos, s_rowkv, st_i);
                 } else if (lin == 2)
                     reduce_gu<DRAFT>(P, l, t, cw, lane, s, ks, tag, st_i);
                 else
                     reduce_residual<DRAFT>(P, lin, l, t, cw, lane, s, ks, tag, st_i);
                 bar_compute();
-                if (ct == 0) {
-                    // one release per reduction, on the counter its consumers poll
-                    if (lin == 1 || lin == 3) red_release_add(ctr(P, l, lin == 1 ? P.cl.res_o : P.cl.res_dn), 1);
-                    if (lin == 0) {
-                        // the attention of every group the tile feeds counts this reduction
-                        int g0, g1;
-                        qkv_tile_groups(P.dm, t, &g0, &g1);
-                        for (int g = g0; g <= g1; ++g) red_release_add(ctr(P, l, P.cl.att_in + g), 1);
-                    }
-                }
+                // one release per reduction, on the counters its consumers poll
+                if (ct == 0) release_item(P, it);
                 if (tr && ct == 0) tr[MK_STAMPS * i + 7] = globaltimer_ns();
             }
         }
@@ -1358,16 +1357,30 @@ void mk_counter_layout(const Dims &dm, int max_nb, CounterLayout *cl) {
     cl->res_dn = cl->res_o + 1;
     cl->att = cl->res_dn + 1;
     cl->att_in = cl->att + max_nb * dm.Hkv;
-    cl->per_layer = cl->att_in + dm.Hkv;
+    cl->att_o = cl->att_in + dm.Hkv;
+    cl->per_layer = cl->att_o + (dm.Hq * dm.d + 255) / 256;
     cl->total = cl->global + dm.nl * cl->per_layer;
 }
 
 // Topologically ordered item list, dealt round-robin over `grid` CTAs (CTA i takes items
 // i, i+grid, ...), so each CTA's list is in dependency order.  Returns items sorted by CTA.
+// Every item carries the one counter it waits for and the counters it adds to once done:
+//   embed row       -> embed counter (target M for layer 0's q|k|v)
+//   q|k|v slice     waits for layer l-1's residual after down (8 tiles x 12 slices at 0.6B) or the
+//                   embeddings; its reduction counts on att_in of each KV group its tile feeds
+//   attention split waits for att_in of its group (every slice of every q, k, v tile of the
+//                   group); the (sequence, group) merge counter orders the split's own merge, and a
+//                   finished merge counts on att_o of the o slice that reads the group
+//   o slice         waits for att_o (every merge of every sequence's groups in the slice); its
+//                   reduction counts on res_o
+//   gate|up slice   waits for res_o (every o tile slice); its reduction writes tagged act words
+//   down slice      waits for nothing (its staging polls the act words); counts on res_dn
+//   final norm row  waits for res_dn of the last layer run.
 void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int> &nsplit, int grid,
-                       std::vector<MKItem> *out, std::vector<int> *off) {
+                       const CounterLayout &cl, std::vector<MKItem> *out, std::vector<int> *off) {
     std::vector<MKItem> all;
-    auto push = [&](uint8_t op, uint8_t lin, int layer, int a, int b, int c) {
+    auto push = [&](uint8_t op, uint8_t lin, int layer, int a, int b, int c, int wait_off, int wait_tgt, int rel0,
+                    int rel1) {
         MKItem it;
         it.op = op;
         it.lin = lin;
@@ -1375,31 +1388,89 @@ void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int
         it.a = a;
         it.b = b;
         it.c = c;
+        it.wait_off = wait_off;
+        it.wait_tgt = wait_tgt;
+        it.rel[0] = rel0;
+        it.rel[1] = rel1;
         all.push_back(it);
     };
-    for (int m = 0; m < pd.M; ++m) push(MK_EMBED, 0, 0, m, 0, 0);
     const int nq = (dm.Hq + 2 * dm.Hkv) * dm.d / TILE_ROWS;
     const int n_main[4] = {nq, dm.H / TILE_ROWS, 2 * dm.I / TILE_ROWS, dm.H / TILE_ROWS};
     const int K[4] = {dm.H, dm.Hq * dm.d, dm.H, dm.I};
-    auto linear = [&](int lin, int l) {
-        const int ks = K[lin] / (mk_slice_atoms(lin, K[lin]) * KT);
-        if (pd.adapter)
-            for (int s = 0; s < ks; ++s) push(MK_LINEAR, lin, l, n_main[lin], s, 0);
-        for (int t = 0; t < n_main[lin]; ++t)
-            for (int s = 0; s < ks; ++s) push(MK_LINEAR, lin, l, t, s, 0);
+    int ks[4];
+    for (int lin = 0; lin < 4; ++lin) ks[lin] = K[lin] / (mk_slice_atoms(lin, K[lin]) * KT);
+    const int grp = dm.Hq / dm.Hkv, qw = dm.Hq * dm.d, kvw = dm.Hkv * dm.d, gw = grp * dm.d;
+    auto ctr = [&](int layer, int o) { return cl.global + layer * cl.per_layer + o; };
+    // KV groups a q|k|v tile feeds
+    auto tile_groups = [&](int t, int *g0, int *g1) {
+        const int f0 = t * TILE_ROWS, f1 = f0 + TILE_ROWS - 1;
+        if (f0 < qw) {
+            *g0 = f0 / gw;
+            *g1 = f1 / gw;
+        } else {
+            const int base = f0 < qw + kvw ? qw : qw + kvw;
+            *g0 = (f0 - base) / dm.d;
+            *g1 = (f1 - base) / dm.d;
+        }
     };
+    // reduced slices an attention item of group g waits for
+    std::vector<int> att_in_tgt(dm.Hkv, 0);
+    for (int t = 0; t < nq; ++t) {
+        int g0, g1;
+        tile_groups(t, &g0, &g1);
+        for (int g = g0; g <= g1; ++g) att_in_tgt[g] += ks[0];
+    }
+    // merges per (sequence, group): every split when the splits sit on distinct CTAs, else the last
+    int merges = 0;
+    for (int bl = 0; bl < pd.nb; ++bl) merges += nsplit[bl] <= grid ? nsplit[bl] : 1;
+    const int o_w = mk_slice_atoms(1, K[1]) * KT;  // o slice width
+    for (int m = 0; m < pd.M; ++m) push(MK_EMBED, 0, 0, m, 0, 0, -1, 0, cl.embed, -1);
     for (int l = 0; l < pd.nl_run; ++l) {
-        linear(0, l);
+        auto linear = [&](int lin, int wait_off, int wait_tgt) {
+            for (int r = 0; r < (pd.adapter ? 1 : 0) + n_main[lin]; ++r) {
+                const int t = pd.adapter ? (r == 0 ? n_main[lin] : r - 1) : r;  // adapter tile first
+                int rel0 = -1, rel1 = -1;
+                if (t < n_main[lin]) {
+                    if (lin == 0) {
+                        int g0, g1;
+                        tile_groups(t, &g0, &g1);
+                        rel0 = ctr(l, cl.att_in + g0);
+                        rel1 = g1 != g0 ? ctr(l, cl.att_in + g1) : -1;
+                    } else if (lin == 1) {
+                        rel0 = ctr(l, cl.res_o);
+                    } else if (lin == 3) {
+                        rel0 = ctr(l, cl.res_dn);
+                    }
+                }
+                for (int sl = 0; sl < ks[lin]; ++sl) push(MK_LINEAR, lin, l, t, sl, 0, wait_off, wait_tgt, rel0, rel1);
+            }
+        };
+        if (l == 0)
+            linear(0, cl.embed, pd.M);
+        else
+            linear(0, ctr(l - 1, cl.res_dn), n_main[3] * ks[3]);
         for (int bl = 0; bl < pd.nb; ++bl)
             for (int g = 0; g < dm.Hkv; ++g)
-                for (int s = 0; s < nsplit[bl]; ++s) push(MK_ATTN, 0, l, bl, g, s);
-        linear(1, l);
-        linear(2, l);
-        linear(3, l);
+                for (int sp = 0; sp < nsplit[bl]; ++sp)
+                    push(MK_ATTN, 0, l, bl, g, sp, ctr(l, cl.att_in + g), att_in_tgt[g], ctr(l, cl.att_o + g * gw / o_w),
+                         -1);
+        // o slice sl reads the heads of the groups g with g * gw / o_w == sl
+        for (int r = 0; r < (pd.adapter ? 1 : 0) + n_main[1]; ++r) {
+            const int t = pd.adapter ? (r == 0 ? n_main[1] : r - 1) : r;
+            for (int sl = 0; sl < ks[1]; ++sl) {
+                int groups = 0;
+                for (int g = 0; g < dm.Hkv; ++g) groups += (g * gw / o_w == sl) ? 1 : 0;
+                push(MK_LINEAR, 1, l, t, sl, 0, ctr(l, cl.att_o + sl), groups * merges,
+                     t < n_main[1] ? ctr(l, cl.res_o) : -1, -1);
+            }
+        }
+        linear(2, ctr(l, cl.res_o), n_main[1] * ks[1]);
+        linear(3, -1, 0);
     }
     for (int bl = 0; bl < pd.nb; ++bl)
         for (int i = pd.ro_first; i < pd.ro_first + pd.ro_count; ++i)
-            push(MK_FINAL, 0, pd.nl_run - 1, bl * pd.ro_count + (i - pd.ro_first), bl * pd.R + i, 0);
+            push(MK_FINAL, 0, pd.nl_run - 1, bl * pd.ro_count + (i - pd.ro_first), bl * pd.R + i, 0,
+                 ctr(pd.nl_run - 1, cl.res_dn), n_main[3] * ks[3], -1, -1);
     off->assign(grid + 1, 0);
     for (size_t i = 0; i < all.size(); ++i) (*off)[i % grid + 1]++;
     for (int c = 0; c < grid; ++c) (*off)[c + 1] += (*off)[c];

@@ -414,7 +414,7 @@ PassDesc block_pass(pbd_ctx *c, int kind) {
 pbd_status upload_schedule(pbd_ctx *c, int kind, const PassDesc &pd, const std::vector<int> &nsplit) {
     std::vector<MKItem> items;
     std::vector<int> off;
-    mk_build_schedule(c->dm, pd, nsplit, c->grid, &items, &off);
+    mk_build_schedule(c->dm, pd, nsplit, c->grid, c->cl, &items, &off);
     if (items.size() > c->items_cap)
         return fail(c, PBD_ERR_CAPACITY, "pass schedule of %zu items exceeds %zu", items.size(), c->items_cap);
     Sched &s = c->sched[kind];
@@ -617,14 +617,19 @@ pbd_status pbd_plan_pass(const pbd_config *cfg, int32_t kind, int32_t batch, con
     tmp.prompt_lens.assign(h_prompt_lens, h_prompt_lens + batch);
     std::vector<MKItem> items;
     std::vector<int> off;
-    mk_build_schedule(tmp.dm, block_pass(&tmp, kind), decode_splits(&tmp), grid, &items, &off);
+    mk_build_schedule(tmp.dm, block_pass(&tmp, kind), decode_splits(&tmp), grid, tmp.cl, &items, &off);
     *h_n = (int32_t)items.size();
     if ((int)items.size() > cap) return fail(nullptr, PBD_ERR_CAPACITY, "%zu items exceed cap %d", items.size(), cap);
     for (size_t i = 0; i < items.size(); ++i) {
-        h_items[4 * i] = items[i].op | (items[i].lin << 8) | (items[i].layer << 16);
-        h_items[4 * i + 1] = items[i].a;
-        h_items[4 * i + 2] = items[i].b;
-        h_items[4 * i + 3] = items[i].c;
+        int32_t *o = h_items + 8 * i;
+        o[0] = items[i].op | (items[i].lin << 8) | (items[i].layer << 16);
+        o[1] = items[i].a;
+        o[2] = items[i].b;
+        o[3] = items[i].c;
+        o[4] = items[i].wait_off;
+        o[5] = items[i].wait_tgt;
+        o[6] = items[i].rel[0];
+        o[7] = items[i].rel[1];
     }
     for (int k = 0; k <= grid; ++k) h_cta_off[k] = off[k];
     return PBD_OK;
@@ -1052,7 +1057,7 @@ pbd_status pbd_check_stalled_pass(pbd_ctx *c, int32_t *h_device_code) {
     const std::vector<int> ns = decode_splits(c);
     std::vector<MKItem> all, items;
     std::vector<int> off;
-    mk_build_schedule(c->dm, pd, ns, 1, &all, &off);  // one CTA: the items in order
+    mk_build_schedule(c->dm, pd, ns, 1, c->cl, &all, &off);  // one CTA: the items in order
     bool dropped = false;
     for (const MKItem &it : all) {
         if (!dropped && it.op == MK_LINEAR && it.lin == 0 && it.layer == 0) {
@@ -1090,7 +1095,7 @@ pbd_status pbd_trace_pass(pbd_ctx *c, int32_t kind, int32_t *h_items, uint64_t *
     const PassDesc pd = block_pass(c, kind);
     std::vector<MKItem> items;
     std::vector<int> off;
-    mk_build_schedule(c->dm, pd, decode_splits(c), c->grid, &items, &off);
+    mk_build_schedule(c->dm, pd, decode_splits(c), c->grid, c->cl, &items, &off);
     if ((int)items.size() > cap) return fail(c, PBD_ERR_CAPACITY, "%zu items exceed cap %d", items.size(), cap);
     CK(launch_build_ids(pd, kind == PK_DRAFT ? 0 : (kind == PK_VERIFY ? 1 : 2), c->s.pending, c->draft_ids, c->D,
                         c->ids, c->st));

@@ -80,10 +80,15 @@ constexpr int MK_STAMPS = 16;
 // One work item of a pass.  MK_LINEAR: lin (0 q|k|v, 1 o, 2 gate|up, 3 down), a = row tile
 // (the adapter tile is the last one), b = 256-wide K slice.  MK_ATTN: a = sequence in the pass,
 // b = KV head, c = 128-key split.  MK_EMBED: a = row.  MK_FINAL: a = read-out index, b = row.
+// Dependencies, worked out on the host: the item waits until counter wait_off (an index into the
+// pass's counters, -1: none) reaches wait_tgt, and once its result is stored it adds one to each
+// counter rel[k] >= 0 (a reduction, an embedded row, an attention merge).
 struct __align__(16) MKItem {
     uint8_t op, lin;
     uint16_t layer;
     int32_t a, b, c;
+    int32_t wait_off, wait_tgt;
+    int32_t rel[2];
 };
 
 // Offsets of the pass's completion counters (ints, zeroed before every pass).
@@ -94,6 +99,7 @@ struct CounterLayout {
     int res_o, res_dn;  // residual tiles finished after o / down
     int att;        // per (sequence, KV head): split items done (+1 once merged)
     int att_in;     // per KV head: reduced q|k|v tile slices that its attention reads
+    int att_o;      // per K slice of the o projection: attention merges of the heads it reads
     int total;
 };
 
@@ -133,7 +139,7 @@ struct MKLaunch {
 int mk_grid_size();
 void mk_counter_layout(const Dims &dm, int max_nb, CounterLayout *cl);
 void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int> &nsplit, int grid,
-                       std::vector<MKItem> *out, std::vector<int> *off);
+                       const CounterLayout &cl, std::vector<MKItem> *out, std::vector<int> *off);
 size_t mk_union_bytes(int bn, int head_dim);
 int mk_slice_atoms(int lin, int K);  // 64-wide K atoms per work item of linear `lin`
 cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st);

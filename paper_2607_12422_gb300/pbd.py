@@ -225,10 +225,11 @@ def make_config(shape, block_D: int, max_batch: int, max_seq_len: int, draft_lay
 
 def pbd_plan_pass(cfg: pbd_config, kind: int, prompt_lens: Sequence[int], max_new: int, grid: int,
                   cap: int = 1 << 20):
-    """(items [n, 4] int32, cta_off [grid + 1] int32) of one pass's schedule, host only."""
+    """(items [n, 8] int32, cta_off [grid + 1] int32) of one pass's schedule, host only: per item
+    {op | lin << 8 | layer << 16, a, b, c, wait counter, wait target, release counters 0, 1}."""
     L = load()
     lens = np.ascontiguousarray(np.asarray(prompt_lens, dtype=np.int32))
-    items = np.zeros((cap, 4), np.int32)
+    items = np.zeros((cap, 8), np.int32)
     off = np.zeros(grid + 1, np.int32)
     n = np.zeros(1, np.int32)
     s = L.pbd_plan_pass(C.byref(cfg), kind, len(lens), lens.ctypes.data, max_new, grid, items.ctypes.data,

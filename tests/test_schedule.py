@@ -107,6 +107,42 @@ def _check(S, items, off, grid, n_layers_run, slice_w):
     assert set(layer[op == OP_LINEAR]) == set(range(n_layers_run))
 
 
+def _check_counters(items, off, grid):
+    """The host-computed waits agree with the releases: every counter an item waits for receives
+    exactly its target of releases, all from items earlier in the list.  Attention splits release
+    once each after merging when a group's splits sit on distinct CTAs, else only the last one."""
+    n = len(items)
+    g = _global_order(off, grid, n)
+    op, lin, layer, a, b, c = _decode(items)
+    w_off, w_tgt, rel = items[:, 4], items[:, 5], items[:, 6:8]
+    att_groups = {}
+    for i in np.nonzero(op == OP_ATTN)[0]:
+        att_groups.setdefault((layer[i], a[i], b[i]), []).append(i)
+    count, last = {}, {}
+    for i in range(n):
+        if op[i] == OP_ATTN:
+            continue
+        for r in rel[i]:
+            if r >= 0:
+                count[r] = count.get(r, 0) + 1
+                last[r] = max(last.get(r, -1), g[i])
+    for idx in att_groups.values():
+        r = rel[idx[0], 0]
+        assert (rel[idx, 0] == r).all() and (rel[idx, 1] == -1).all()
+        count[r] = count.get(r, 0) + (len(idx) if len(idx) <= grid else 1)
+        last[r] = max(last.get(r, -1), max(g[idx]))
+    waits = 0
+    for i in range(n):
+        if w_off[i] < 0:
+            assert op[i] == OP_EMBED or (op[i] == OP_LINEAR and lin[i] == 3), i  # down polls act words
+            continue
+        waits += 1
+        assert count.get(w_off[i], 0) == w_tgt[i], (i, "waits for", w_tgt[i], "releases of", w_off[i],
+                                                    "which receives", count.get(w_off[i], 0))
+        assert last[w_off[i]] < g[i], (i, "waits for a release later in the list")
+    assert waits > 0
+
+
 CASES = [
     ("tiny", synth.TINY, 16, [64], 64),
     ("tiny-b4", synth.TINY, 16, [64, 40, 17, 100], 64),
@@ -126,6 +162,7 @@ def test_schedule_is_deadlock_free(case, kind, grid):
     items, off = pbd.pbd_plan_pass(cfg, kind, lens, G, grid)
     slice_w = [256, 256, 512 if S.hidden % 512 == 0 else 256, 256]
     _check(S, items, off, grid, S.n_layers, slice_w)
+    _check_counters(items, off, grid)
     op, lin, layer, a, b, c = _decode(items)
     rows = len(lens) * (1 if kind == 2 else D + 1)
     assert (op == OP_EMBED).sum() == rows
@@ -143,6 +180,7 @@ def test_early_exit_schedule(E):
     cfg = pbd.make_config(S, 16, 1, 1024, draft_layers=E)
     items, off = pbd.pbd_plan_pass(cfg, 0, [512], 256, 152)
     _check(S, items, off, 152, E, [256, 256, 512, 256])
+    _check_counters(items, off, 152)
     # the verify pass still runs every layer
     items_v, off_v = pbd.pbd_plan_pass(cfg, 1, [512], 256, 152)
     _check(S, items_v, off_v, 152, S.n_layers, [256, 256, 512, 256])
@@ -170,6 +208,28 @@ def _redeal(all_items, grid):
         out[fill[i % grid]] = all_items[i]
         fill[i % grid] += 1
     return out, off
+
+
+@pytest.mark.parametrize("mistake", ["target-low", "release-dropped", "wrong-counter"])
+def test_counter_check_catches_planted_mistakes(mistake):
+    S = synth.QWEN3_0_6B
+    cfg = pbd.make_config(S, 16, 1, 1024)
+    items, off = pbd.pbd_plan_pass(cfg, 1, [512], 256, 152)
+    _check_counters(items, off, 152)
+    bad = items.copy()
+    op, lin, layer, a, b, c = _decode(bad)
+    if mistake == "target-low":  # an o slice that would start one merge early
+        i = int(np.nonzero((op == OP_LINEAR) & (lin == 1) & (layer == 3))[0][0])
+        bad[i, 5] -= 1
+    elif mistake == "release-dropped":  # a q|k|v reduction that never counts
+        i = int(np.nonzero((op == OP_LINEAR) & (lin == 0) & (layer == 2) & (a == 0))[0][0])
+        bad[i, 6] = -1
+    else:  # a down reduction counting on the o counter
+        i = int(np.nonzero((op == OP_LINEAR) & (lin == 3) & (layer == 5))[0][0])
+        j = int(np.nonzero((op == OP_LINEAR) & (lin == 1) & (layer == 5))[0][0])
+        bad[i, 6] = bad[j, 6]
+    with pytest.raises(AssertionError):
+        _check_counters(bad, off, 152)
 
 
 @pytest.mark.parametrize("mistake", ["attention-before-qkv", "down-before-gate-up", "slices-apart"])
