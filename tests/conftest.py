@@ -35,3 +35,19 @@ def tiny_zeroB():
     ad = synth.gen_adapter(S, zero_B=True)
     prompt = synth.gen_prompts(S, [64])[0]
     return dict(shape=S, base=base, adapter=ad, prompt=prompt, model=oracle.OracleModel(S, base, ad))
+
+
+def pytest_terminal_summary(terminalreporter, exitstatus, config):
+    """The measured GPU-vs-oracle logit differences and near-ties of the parity tests that ran."""
+    import _parity
+    lines = _parity.summary_lines()
+    if not lines:
+        return
+    terminalreporter.write_sep("-", "parity measurements")
+    for line in lines:
+        terminalreporter.write_line(line)
+    path = os.environ.get("PBD_PARITY_JSON")
+    if path:
+        import json
+        with open(path, "w") as f:
+            json.dump(_parity.RECORDS, f, indent=1)

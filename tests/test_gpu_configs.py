@@ -1,25 +1,21 @@
 """Full-size parity against the CPU oracle on the long-context, batched and block-size
-workloads of the Qwen3-0.6B shape (28 layers, vocab 151936, rank 16):
+workloads of the Qwen3-0.6B shape (28 layers, vocab 151936, rank 16), in lockstep over several
+speculative rounds (see _parity.py for what is compared and recorded):
 
-- 4096-token prompt, D = 16: one speculative round in lockstep;
-- batch of 8 ragged prompts (420..1757 tokens), D = 16: one batched round, the three
-  shortest sequences compared with their own oracle runs (the others are tied to them by
-  the batch-invariance test of the 0.6B suite);
-- 1024-token prompt, D in {4, 32} (the block-size sweep): one round in lockstep each.
-
-In a round, the draft logits, then the verify logits of the GPU's own drafts, are compared
-with the oracle; ids must equal the oracle's argmax up to ties inside the tolerance, and
-the accepted length is recomputed from the GPU's ids by the oracle's rule.  The tolerance
-is the one of the 0.6B lockstep test: twice the disagreement of two valid oracles (fp32
-and fp64 accumulation) on the same inputs, at least 3e-2 and never above 0.1."""
+- 4096-token prompt, D = 16: three rounds;
+- batch of 8 ragged prompts (420..1757 tokens), D = 16: three batched rounds, every sequence
+  compared with its own oracle run (the longest ones exercise the deepest split-KV merges);
+- 1024-token prompt, D in {4, 8, 16, 32} (the block-size sweep): three rounds each.
+"""
 import numpy as np
 import pytest
 
+import _parity
 import oracle
 from paper_2607_12422_gb300 import synth
 
 pytestmark = pytest.mark.gpu
-TOL = 3e-2
+ROUNDS = 3
 
 
 @pytest.fixture(scope="module")
@@ -34,114 +30,50 @@ def cenv():
                 m64=oracle.OracleModel(S, base, ad, acc="f64acc"))
 
 
-def _check_ids(ids, ref_logits, tol):
-    ids = np.asarray(ids).reshape(-1)
-    ref_logits = ref_logits.reshape(len(ids), -1)
-    for j, t in enumerate(ids):
-        best = int(np.argmax(ref_logits[j]))
-        if t != best:
-            assert ref_logits[j][best] - ref_logits[j][t] <= tol, (j, int(t), best)
-
-
-def _tol(a, b):
-    return min(0.1, max(TOL, 2 * float(np.abs(a - b).max())))
-
-
-class _Seq:
-    """One sequence on the two oracles (fp32 and fp64 accumulation) after its prefill."""
-
-    def __init__(self, cenv, prompt, D):
-        P = len(prompt)
-        cap = P + 2 * (D + 1)
-        self.m, self.m64, self.D, self.L = cenv["m"], cenv["m64"], D, P
-        self.cache, self.p, self.lg0 = self.m.prefill(prompt, cap, want_logits=True)
-        self.cache64, _, _ = self.m64.prefill(prompt, cap)
-
-    def draft(self):
-        rows = [self.p] + [-1] * self.D
-        _, od, _ = self.m.forward(self.cache, self.L, rows, True, oracle.MASK_BLOCK_DRAFT, 0, self.D, want_logits=True)
-        _, od64, _ = self.m64.forward(self.cache64, self.L, rows, True, oracle.MASK_BLOCK_DRAFT, 0, self.D,
-                                      want_logits=True)
-        return od, _tol(od, od64)
-
-    def verify(self, drafts):
-        rows = [self.p] + list(drafts)
-        _, ov, _ = self.m.forward(self.cache, self.L, rows, False, oracle.MASK_CAUSAL, 0, self.D + 1, want_logits=True)
-        _, ov64, _ = self.m64.forward(self.cache64, self.L, rows, False, oracle.MASK_CAUSAL, 0, self.D + 1,
-                                      want_logits=True)
-        return ov, _tol(ov, ov64)
-
-
-def _round(eng, seqs):
-    """One speculative round of the engine's batch; seqs maps a batch index to its oracle."""
-    d_ids, d_lg = eng.pbd_draft_block(want_logits=True)
-    for b, sq in seqs.items():
-        od, tol = sq.draft()
-        assert np.abs(d_lg[b].cpu().numpy() - od).max() <= tol, b
-        _check_ids(d_ids[b].cpu().numpy(), od, tol)
-    v_ids, v_lg = eng.pbd_verify_block(want_logits=True)
-    n_gpu = eng.pbd_accept_commit()
-    for b, sq in seqs.items():
-        drafts = [int(t) for t in d_ids[b].cpu()]
-        ov, tol = sq.verify(drafts)
-        assert np.abs(v_lg[b].cpu().numpy() - ov).max() <= tol, b
-        verify = [int(t) for t in v_ids[b].cpu()]
-        _check_ids(verify, ov, tol)
-        assert int(n_gpu[b]) == oracle.accept_length(drafts, verify), b
-
-
-def _start(eng, prompts, seqs, max_new):
-    """Prefill; a sequence whose first token is a near-tie between GPU and oracle (checked) leaves
-    the comparison, since lockstep needs a common start."""
-    first = eng.pbd_prefill(prompts, max_new=max_new)
-    for b in list(seqs):
-        if int(first[b]) != seqs[b].p:
-            _check_ids([int(first[b])], seqs[b].lg0[None], 0.1)
-            del seqs[b]
-    if not seqs:
-        pytest.skip("every compared sequence starts on a near-tie")
-
-
-def test_long_context_4096_round(cenv):
+def test_long_context_4096_rounds(cenv):
     W = synth.WORKLOADS["qwen3-0.6b-b1-d16-p4096-g512"]
     prompt = synth.gen_prompts(W.shape, list(W.prompt_lens))[0]
     eng = cenv["pbd"].Engine(cenv["S"], cenv["base"], cenv["ad"], block_D=W.block_D, max_batch=1,
-                             max_seq_len=len(prompt) + 64)
-    seqs = {0: _Seq(cenv, prompt, W.block_D)}
-    _start(eng, [prompt], seqs, 32)
-    _round(eng, seqs)
+                             max_seq_len=len(prompt) + 96)
+    seqs = {0: _parity.Seq(cenv["m"], cenv["m64"], prompt, W.block_D, ROUNDS)}
+    _parity.start(eng, [prompt], seqs, 64, W.name)
+    _parity.rounds(eng, seqs, ROUNDS, W.name)
     eng.close()
 
 
-def test_batch8_ragged_round(cenv):
+def test_batch8_ragged_rounds(cenv):
     W = synth.WORKLOADS["qwen3-0.6b-b8-d16-p256to2048-g256"]
     prompts = synth.gen_prompts(W.shape, list(W.prompt_lens))
     eng = cenv["pbd"].Engine(cenv["S"], cenv["base"], cenv["ad"], block_D=W.block_D, max_batch=8,
-                             max_seq_len=max(W.prompt_lens) + 64)
-    shortest = sorted(range(len(prompts)), key=lambda b: len(prompts[b]))[:3]
-    seqs = {b: _Seq(cenv, prompts[b], W.block_D) for b in shortest}
-    _start(eng, prompts, seqs, 32)
-    _round(eng, seqs)
+                             max_seq_len=max(W.prompt_lens) + 96)
+    seqs = {b: _parity.Seq(cenv["m"], cenv["m64"], prompts[b], W.block_D, ROUNDS) for b in range(len(prompts))}
+    _parity.start(eng, prompts, seqs, 64, W.name)
+    _parity.rounds(eng, seqs, ROUNDS, W.name)
     eng.close()
 
 
 @pytest.fixture(scope="module")
 def sweep(cenv):
-    """The block-size sweep's 1024-token prompt, prefilled once on both oracles.  A round
-    writes only slots >= the prompt length, so every block size starts from the same cache."""
+    """The block-size sweep's 1024-token prompt, prefilled once on both oracles; each block size
+    continues from a copy of that cache."""
     W = synth.WORKLOADS["qwen3-0.6b-b1-p1024-dsweep-forced"]
     prompt = synth.gen_prompts(W.shape, list(W.prompt_lens))[0]
-    return W, prompt, _Seq(cenv, prompt, max(W.D_sweep))
+    return W, prompt, _parity.Seq(cenv["m"], cenv["m64"], prompt, max(W.D_sweep), ROUNDS)
 
 
-@pytest.mark.parametrize("D", [4, 32])
-def test_block_size_sweep_round(cenv, sweep, D):
-    W, prompt, sq = sweep
+@pytest.mark.parametrize("D", [4, 8, 16, 32])
+def test_block_size_sweep_rounds(cenv, sweep, D):
+    W, prompt, base_sq = sweep
     assert D in W.D_sweep
-    sq.D = D
-    eng = cenv["pbd"].Engine(cenv["S"], cenv["base"], cenv["ad"], block_D=D, max_batch=1,
-                             max_seq_len=len(prompt) + 96)
+    P = len(prompt)
+    sq = _parity.Seq.__new__(_parity.Seq)
+    sq.m, sq.m64, sq.D, sq.L, sq.p, sq.lg0 = base_sq.m, base_sq.m64, D, P, base_sq.p, base_sq.lg0
+    cap = P + (ROUNDS + 1) * (max(W.D_sweep) + 1)
+    sq.cache, sq.cache64 = sq.m.new_cache(cap), sq.m64.new_cache(cap)
+    base_sq.cache.copy_to(sq.cache, P)
+    base_sq.cache64.copy_to(sq.cache64, P)
+    eng = cenv["pbd"].Engine(cenv["S"], cenv["base"], cenv["ad"], block_D=D, max_batch=1, max_seq_len=P + 160)
     seqs = {0: sq}
-    _start(eng, [prompt], seqs, 32)
-    _round(eng, seqs)
+    _parity.start(eng, [prompt], seqs, 96, "%s-D%d" % (W.name, D))
+    _parity.rounds(eng, seqs, ROUNDS, "%s-D%d" % (W.name, D))
     eng.close()

@@ -6,6 +6,7 @@ rows bit for bit)."""
 import numpy as np
 import pytest
 
+import _parity
 import oracle
 from paper_2607_12422_gb300 import synth
 
@@ -61,6 +62,20 @@ def test_round_matches_oracle(env):
     assert int(L[0]) == P + int(n[0]) + 1
     assert int(pend[0]) == verify[int(n[0])]
     assert int(n_out[0]) == 1 + int(n[0]) + 1
+
+
+def test_lockstep_rounds_strict(env):
+    """Eight rounds in lockstep at the stated tolerance of 3e-2 with no widening: every verify id
+    and every generated token equals the oracle's argmax exactly (no near-tie allowed on the tiny
+    model); draft ids may differ only inside 3e-2 (recorded)."""
+    eng, m, prompt = env["eng"], env["model"], env["prompts"][0]
+    seqs = {0: _parity.Seq(m, None, prompt, D, 8)}
+    _parity.start(eng, [prompt], seqs, 64, "tiny-b1-d16-p64-g64")
+    n0 = len(_parity.RECORDS)
+    _parity.rounds(eng, seqs, 8, "tiny-b1-d16-p64-g64")
+    new = _parity.RECORDS[n0:]
+    assert all(r["bound"] == TOL for r in new)
+    assert sum(r["id_mismatches"] for r in new if r["pass_kind"] == "verify") == 0
 
 
 def test_generate_equals_oracle_greedy(env):
