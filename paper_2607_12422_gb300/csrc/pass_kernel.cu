@@ -80,6 +80,11 @@ __device__ __forceinline__ void st_relaxed_u64(unsigned long long *p, unsigned l
     asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(v));
 }
 __device__ __forceinline__ bool tag_is(unsigned long long w, uint32_t tag) { return (uint32_t)(w >> 32) == tag; }
+// one tagged word (value in the low half, tag in the high half), single-copy atomic
+__device__ __forceinline__ void st_tagged(unsigned long long *p, uint32_t v, uint32_t tag) {
+    asm volatile("{\n\t.reg .b64 w;\n\tmov.b64 w, {%1, %2};\n\tst.relaxed.gpu.global.b64 [%0], w;\n\t}" ::"l"(p),
+                 "r"(v), "r"(tag));
+}
 // 16-byte load, single-copy atomic per 64-bit element
 __device__ __forceinline__ void ld_relaxed_2u64(const unsigned long long *p, unsigned long long &a,
                                                 unsigned long long &b) {
@@ -992,6 +997,331 @@ __device__ __forceinline__ void release_item(const MKParams &P, const MKItem &it
 
 // ------------------------------------------------------------------ the kernel
 
+// Per-CTA shared state of the pass kernel (static shared memory).
+struct CtaState {
+    uint64_t full[MAX_SLOT], empty[MAX_SLOT], b_full[2], b_empty, acc_full, att_bar, mma_drain;
+    uint32_t tmem_slot;
+    // compute-group flags: each is written by thread 0 and read by all after a barrier, and is
+    // not written again before every thread has passed at least one more barrier
+    int flag, red, ok;
+    uint32_t tag;  // this pass's partial-sum tag
+    float rms[MAX_ROWS];
+    int phys[2][ATT_SPLIT / PAGE];  // page ids of attention stages 0 and 1
+    // per pass row: position (-1 beyond the RoPE table) and KV slot (page << 4 | slot; -1 beyond
+    // the reserved pages)
+    int rowpos[MAX_ROWS], rowkv[MAX_ROWS];
+};
+
+// ---- warp 0 lane 0: weight producer.  Walks the CTA's linear items ahead of the others and
+// streams their 128 x 64 weight tiles into the ring (1-D bulk TMA, L2 evict-first); weights depend
+// on nothing, so the ring fills across phase boundaries.
+__device__ __noinline__ void run_producer(const MKParams &P, const MKItem *my, int n_my, uint8_t *ring, CtaState &S) {
+    const uint64_t pol = l2_policy_evict_first();
+    uint32_t kt = 0;
+#pragma unroll 1
+    for (int i = 0; i < n_my && !aborted(P); ++i) {
+        const MKItem it = my[i];
+        if (it.op != MK_LINEAR) continue;
+        const int lin = it.lin;
+        const bool lt = it.a >= P.n_main[lin] / TILE_ROWS;
+        const uint32_t bytes = lt ? (uint32_t)P.lora_rows[lin] * 128u : (uint32_t)TILE_BYTES;
+        const int kts = P.K[lin] / KT;
+        const uint8_t *src =
+            P.wt[lin] + P.wt_stride[lin] * it.layer + ((size_t)it.a * kts + (size_t)it.b * P.katoms[lin]) * TILE_BYTES;
+        bool ok = true;
+#pragma unroll 1
+        for (int j = 0; j < P.katoms[lin]; ++j, ++kt) {
+            const int slot = kt % P.nslot;
+            if (kt >= (uint32_t)P.nslot && !mbar_wait_mk(&S.empty[slot], ((kt / P.nslot) - 1) & 1, P, DEV_TIMEOUT_SLOT)) {
+                ok = false;
+                break;
+            }
+            mbar_arrive_expect_tx(&S.full[slot], bytes);
+            bulk_g2s(ring + (size_t)slot * TILE_BYTES, src + (size_t)j * TILE_BYTES, bytes, &S.full[slot], pol);
+        }
+        if (!ok) break;
+    }
+    if (aborted(P))  // the last nslot tiles issued may still be in flight: let them land
+#pragma unroll 1
+        for (uint32_t h = kt > (uint32_t)P.nslot ? kt - P.nslot : 0; h < kt; ++h)
+            drain_wait(&S.full[h % P.nslot], (h / P.nslot) & 1);
+}
+
+// ---- warp 1 lane 0: MMA issuer.  Per linear item, 4 (or 8) x 4 tcgen05.mma (128 x bn x 16,
+// bf16 -> fp32) into the TMEM accumulator; frees ring slots with tcgen05.commit.
+__device__ __noinline__ void run_mma(const MKParams &P, const MKItem *my, int n_my, uint8_t *ring, uint8_t *uni,
+                                     uint32_t tmem, CtaState &S) {
+    const uint32_t idesc = idesc_bf16_f32(128, P.bn);
+    uint32_t kt = 0, li = 0, l8 = 0;
+#pragma unroll 1
+    for (int i = 0; i < n_my; ++i) {
+        const MKItem it = my[i];
+        if (it.op != MK_LINEAR) continue;
+        const int na = P.katoms[it.lin];
+        if (!mbar_wait_mk(&S.b_full[0], li & 1, P, DEV_TIMEOUT_LOAD)) break;
+        tc_fence_after();
+        bool ok = true;
+#pragma unroll 1
+        for (int j = 0; j < na; ++j, ++kt) {
+            if (j == HALF_ATOMS) {
+                // second half of a wide slice: its operand is staged after the first half's reads
+                // completed (same area) or was staged with it
+                if (!P.b_dbl) mma_commit(&S.b_empty);
+                if (!mbar_wait_mk(&S.b_full[1], l8 & 1, P, DEV_TIMEOUT_LOAD)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+            }
+            const int slot = kt % P.nslot;
+            if (!mbar_wait_mk(&S.full[slot], (kt / P.nslot) & 1, P, DEV_TIMEOUT_LOAD)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const uint64_t ad = sw128_kmajor_desc(ring + (size_t)slot * TILE_BYTES);
+            const int bj = (P.b_dbl || j < HALF_ATOMS) ? j : j - HALF_ATOMS;
+            const uint64_t bd = sw128_kmajor_desc(uni + (size_t)bj * P.bn * 128);
+#pragma unroll
+            for (int kk = 0; kk < KT / 16; ++kk)
+                mma_bf16_ss(tmem, ad + 2ull * kk, bd + 2ull * kk, idesc, (j | kk) != 0 ? 1u : 0u);
+            mma_commit(&S.empty[slot]);
+        }
+        if (!ok) break;
+        mma_commit(&S.acc_full);
+        ++li;
+        if (na > HALF_ATOMS) ++l8;
+    }
+    if (aborted(P)) {
+        // every MMA issued so far completes before TMEM and the operands are released
+        mma_commit(&S.mma_drain);
+        drain_wait(&S.mma_drain, 0);
+    }
+}
+
+// ---- compute group: final RMSNorm of one read-out row (the lm_head's input)
+__device__ __noinline__ void item_final(const MKParams &P, const MKItem &it, int ct, CtaState &S) {
+    const int r = it.a, m = it.b;
+    if (ct == 0) S.rms[0] = row_rms(P, m);
+    bar_compute();
+    const float rs = S.rms[0];
+#pragma unroll 1
+    for (int c8 = ct; c8 < P.dm.H / 8; c8 += CT) {
+        uint4 hv = __ldcg(reinterpret_cast<const uint4 *>(P.h + (size_t)m * P.dm.H) + c8);
+        const uint4 gv = __ldg(reinterpret_cast<const uint4 *>(P.final_norm) + c8);
+        __nv_bfloat162 *h2 = reinterpret_cast<__nv_bfloat162 *>(&hv);
+        const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(&gv);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float2 f = __bfloat1622float2(h2[e]);
+            h2[e] = __hmul2(g2[e], __floats2bfloat162_rn(__fmul_rn(f.x, rs), __fmul_rn(f.y, rs)));
+        }
+        reinterpret_cast<uint4 *>(P.x_ro + (size_t)r * P.dm.H)[c8] = hv;
+    }
+}
+
+// ---- compute group: one attention split item (pages, split, merge).  Returns false on abort.
+template <bool DRAFT, int DH>
+__device__ __noinline__ bool item_attn(const MKParams &P, const MKItem &it, bool active, uint8_t *uni, CtaState &S,
+                                       uint32_t &ai, int ct, int cw, int lane, unsigned long long *st) {
+    const int bl = it.a, g = it.b, s = it.c;
+    if (active) {
+        if (ct == 0) {
+            attn_pages(P, it.layer, bl, g, s, 1, uni, &S.att_bar, S.phys[1]);
+            stamp_at(st, 8);
+        }
+        attn_split<DH, DRAFT>(P, it.layer, bl, g, s, uni, &S.att_bar, ai & 1, ct, cw, lane, st);
+        ++ai;
+    }
+    bar_compute();
+    if (ct == 0) stamp_at(st, 2);
+    // merge: when the (sequence, head)'s splits fit on distinct CTAs, every split waits for the
+    // others and merges pairs s, s + nsplit, ...; otherwise the last one merges all
+    int *c = ctr(P, it.layer, P.cl.att + bl * P.dm.Hkv + g);
+    const int nsp = P.nsplit[bl];
+    const bool shared_merge = att_shared_merge(nsp);
+    if (ct == 0) {
+        if (shared_merge) {
+            red_release_add(c, 1);
+            S.ok = spin_until(c, nsp, P) ? 1 : 0;
+            S.red = 1;
+        } else {
+            S.red = (atom_acq_rel_add(c, 1) == nsp - 1) ? 1 : 0;
+            S.ok = 1;
+        }
+        stamp_at(st, 6);
+        stamp_at(st, 7);
+    }
+    bar_compute();
+    if (!S.ok) return false;
+    if (S.red) {
+        const int p0 = shared_merge ? s : 0, pstep = shared_merge ? nsp : 1;
+        attn_combine<DH>(P, bl, g, cw, lane, p0, pstep, st);
+        bar_compute();
+        if (ct == 0) {
+            release_item(P, it);  // counts on the o slice that reads the group
+            stamp_at(st, 7);
+        }
+    }
+    return true;
+}
+
+// ---- compute group: one linear slice item: stage the activation operand (warp 1 then issues the
+// MMAs), read the accumulator out as tagged partial sums, and reduce this CTA's share of the tile's
+// rows.  The tile's K slices are consecutive items of the round-robin schedule, so they sit on
+// distinct CTAs that all reach them: each CTA stores its tagged slice partials, then reduces rows
+// s, s + ks, ... of the tile (s = its slice), reading the other slices' partials as they arrive.
+// The adapter tile's partials are summed by the main tiles' reducers themselves.  Returns false
+// on abort.
+template <bool DRAFT, int DH>
+__device__ __noinline__ bool item_linear(const MKParams &P, const MKItem &it, uint8_t *uni, uint32_t tmem, CtaState &S,
+                                         uint32_t &li, uint32_t &l8, int ct, int cw, int lane, int warp,
+                                         unsigned long long *st) {
+    const int lin = it.lin, l = it.layer, t = it.a, s = it.b;
+    const int na = P.katoms[lin];
+    if (na <= HALF_ATOMS) {
+        if (lin == 3)
+            build_b_act(P, s, uni, ct, S.tag + l, st);
+        else
+            build_b(P, lin, l, s, uni, S.rms, ct, 0, true, st);
+        fence_proxy_async();
+        bar_compute();
+        if (ct == 0) mbarrier_arrive_one(&S.b_full[0]);
+    } else {
+        // wide slice in two halves: when both fit, the first half's MMAs run while the second is
+        // staged; else the second goes through the same area after the first half's reads
+        build_b(P, lin, l, s, uni, S.rms, ct, 0, true, st);
+        fence_proxy_async();
+        bar_compute();
+        if (ct == 0) {
+            mbarrier_arrive_one(&S.b_full[0]);
+            if (!P.b_dbl) S.ok = mbar_wait_mk(&S.b_empty, l8 & 1, P, DEV_TIMEOUT_MMA) ? 1 : 0;
+        }
+        if (!P.b_dbl) {
+            bar_compute();
+            if (!S.ok) return false;
+        }
+        build_b(P, lin, l, s, uni + (P.b_dbl ? (size_t)HALF_ATOMS * P.bn * 128 : 0), S.rms, ct, HALF_ATOMS, false,
+                nullptr);
+        fence_proxy_async();
+        bar_compute();
+        if (ct == 0) mbarrier_arrive_one(&S.b_full[1]);
+        ++l8;
+    }
+    if (ct == 0) stamp_at(st, 4);
+    const bool lt = t >= P.n_main[lin] / TILE_ROWS;
+    const uint32_t tag = S.tag + l;
+    if (warp >= 4) {
+        // epilogue: warp 4 + q reads TMEM lanes 32q..32q+31 (the tile's weight rows), 32 token
+        // columns at a time, and stores them as tagged partial sums
+        const int quarter = warp - 4;
+        const bool have = mbar_wait_mk(&S.acc_full, li & 1, P, DEV_TIMEOUT_MMA);
+        if (warp == 4 && lane == 0) stamp_at(st, 5);
+        tc_fence_after();
+        const int row = quarter * 32 + lane;
+        if (have) {
+            // eight token columns per TMEM load (a warp-wide access: every lane takes part)
+            const bool mine = row < (lt ? P.lora_rows[lin] : TILE_ROWS);
+            const int n_total = P.n_main[lin] + P.lora_rows[lin];
+            unsigned long long *d = P.part[lin] + (size_t)s * P.part_rows * n_total + t * TILE_ROWS + row;
+            const uint32_t taddr = tmem + ((uint32_t)(quarter * 32) << 16);
+#pragma unroll 1
+            for (int c0 = 0; c0 < P.pd.M; c0 += 8) {
+                uint32_t v[8];
+                tmem_ld_8cols(taddr + (uint32_t)c0, v);
+                tmem_ld_wait();
+                const int nc = mine ? min(8, P.pd.M - c0) : 0;
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    if (j < nc) st_tagged(d, v[j], tag);
+                    d += n_total;
+                }
+            }
+        }
+        tc_fence_before();
+    }
+    ++li;
+    bar_compute();
+    if (ct == 0) {
+        stamp_at(st, 2);
+        stamp_at(st, 6);
+    }
+    if (lt) {
+        if (ct == 0) stamp_at(st, 7);
+        return true;
+    }
+    const int ks = P.ks[lin];
+    if (lin == 0)
+        reduce_qkv<DH, DRAFT>(P, l, t, cw, lane, s, ks, tag, S.rowpos, S.rowkv, st);
+    else if (lin == 2)
+        reduce_gu<DRAFT>(P, l, t, cw, lane, s, ks, tag, st);
+    else
+        reduce_residual<DRAFT>(P, lin, l, t, cw, lane, s, ks, tag, st);
+    bar_compute();
+    // one release per reduction, on the counters its consumers poll
+    if (ct == 0) {
+        release_item(P, it);
+        stamp_at(st, 7);
+    }
+    return true;
+}
+
+// ---- compute group (warps 2-7): dependency waits, operand staging, epilogues, reductions,
+// attention; the attention's cached pages are requested by thread CT_PAGES while thread 0 polls
+// the item's inputs
+template <bool DRAFT, int DH>
+__device__ __noinline__ void run_compute(const MKParams &P, const MKItem *my, int n_my, uint8_t *uni, uint32_t tmem,
+                                         CtaState &S, int tid) {
+    const int ct = tid - 64, cw = ct >> 5, lane = tid & 31, warp = tid >> 5;
+    uint32_t li = 0, ai = 0, l8 = 0;
+    unsigned long long *tr = P.trace ? P.trace + (size_t)MK_STAMPS * P.cta_off[blockIdx.x] : nullptr;
+    bool att_pend = false;  // (thread CT_PAGES) pages requested for a split that has not waited
+#pragma unroll 1
+    for (int i = 0; i < n_my; ++i) {
+        const MKItem it = my[i];
+        unsigned long long *st = tr ? tr + MK_STAMPS * i : nullptr;
+        if (tr && ct == 0) {
+            const unsigned long long now = globaltimer_ns();
+            if (i > 0) tr[MK_STAMPS * (i - 1) + 3] = now;
+            st[0] = now;
+        }
+        const bool att_active = it.op == MK_ATTN && it.c * ATT_SPLIT < P.L[P.pd.b0 + it.a] + P.pd.R;
+        if (att_active && ct == CT_PAGES) {
+            // pages below the cached length do not depend on this pass: fetch them now (the
+            // barrier after the input wait orders this before the split's arrival)
+            attn_pages(P, it.layer, it.a, it.b, it.c, 0, uni, &S.att_bar, S.phys[0]);
+            att_pend = true;
+        }
+        if (ct == 0) S.flag = wait_deps(P, it) ? 1 : 0;
+        bar_compute();
+        if (!S.flag) break;
+        if (ct == 0 && st) st[1] = st[2] = globaltimer_ns();
+        bool ok = true;
+        if (it.op == MK_LINEAR) {
+            ok = item_linear<DRAFT, DH>(P, it, uni, tmem, S, li, l8, ct, cw, lane, warp, st);
+        } else if (it.op == MK_ATTN) {
+            ok = item_attn<DRAFT, DH>(P, it, att_active, uni, S, ai, ct, cw, lane, st);
+            if (att_active) att_pend = false;
+        } else if (it.op == MK_EMBED) {
+            do_embed(P, it.a, cw, lane);
+            bar_compute();
+            if (ct == 0) release_item(P, it);
+        } else {
+            item_final(P, it, ct, S);
+        }
+        if (!ok) break;
+    }
+    if (tr && ct == 0 && n_my > 0) tr[MK_STAMPS * (n_my - 1) + 3] = globaltimer_ns();
+    if (ct == CT_PAGES && att_pend) {
+        // the pass ended before the split waited for its pages: complete the phase's arrival and
+        // let the copies land (bounded) before the shared memory is released
+        mbarrier_arrive_one(&S.att_bar);
+        const uint64_t t0 = globaltimer_ns();
+        while (!mbar_try_wait(smem_u32(&S.att_bar), ai & 1) && globaltimer_ns() - t0 < WAIT_LIMIT_NS) {
+        }
+    }
+}
+
 // DRAFT: the adapter-on pass with the block-diffusion mask; otherwise adapter off and causal.
 // One instantiation per kind keeps each kernel's code and registers to what that pass runs.
 template <bool DRAFT, int DH>
@@ -1000,47 +1330,36 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *ring = base;
     uint8_t *uni = base + P.ring_bytes;  // activation tile / attention staging
-    __shared__ __align__(8) uint64_t full[MAX_SLOT], empty[MAX_SLOT], b_full[2], b_empty, acc_full, att_bar, mma_drain;
-    __shared__ uint32_t tmem_slot;
-    // compute-group flags: each is written by thread 0 and read by all after a barrier, and is
-    // not written again before every thread has passed at least one more barrier
-    __shared__ int s_flag, s_red, s_ok;
-    __shared__ uint32_t s_tag;  // this pass's partial-sum tag
-    __shared__ float s_rms[MAX_ROWS];
-    __shared__ int s_phys[2][ATT_SPLIT / PAGE];  // page ids of attention stages 0 and 1
-    // per pass row: position (-1 beyond the RoPE table) and KV slot (page << 4 | slot; -1 beyond
-    // the reserved pages)
-    __shared__ int s_rowpos[MAX_ROWS], s_rowkv[MAX_ROWS];
-
+    __shared__ CtaState S;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const MKItem *my = P.items + P.cta_off[blockIdx.x];
     const int n_my = P.cta_off[blockIdx.x + 1] - P.cta_off[blockIdx.x];
 
     if (tid == 0) {
         // the previous pass on this stream has finished: its counter advance is visible. Layer l
-        // of this pass tags its partials s_tag + l; the buffers are reused by every layer and
+        // of this pass tags its partials S.tag + l; the buffers are reused by every layer and
         // pass, so a tag identifies both (acquire: read before the arrival below)
-        s_tag = (uint32_t)ld_acquire(P.epoch) + 1u;
+        S.tag = (uint32_t)ld_acquire(P.epoch) + 1u;
         atomicAdd(P.cnt + MK_STARTED, 1);
         for (int i = 0; i < P.nslot; ++i) {
-            mbar_init(&full[i], 1);
-            mbar_init(&empty[i], 1);
+            mbar_init(&S.full[i], 1);
+            mbar_init(&S.empty[i], 1);
         }
-        mbar_init(&b_full[0], 1);
-        mbar_init(&b_full[1], 1);
-        mbar_init(&b_empty, 1);
-        mbar_init(&acc_full, 1);
-        mbar_init(&att_bar, 1);
-        mbar_init(&mma_drain, 1);
+        mbar_init(&S.b_full[0], 1);
+        mbar_init(&S.b_full[1], 1);
+        mbar_init(&S.b_empty, 1);
+        mbar_init(&S.acc_full, 1);
+        mbar_init(&S.att_bar, 1);
+        mbar_init(&S.mma_drain, 1);
         prefetch_tensormap(&P.kmap);
         prefetch_tensormap(&P.vmap);
         fence_mbarrier_init();
     }
-    if (warp == 0) tmem_alloc(&tmem_slot, P.tmem_cols);
+    if (warp == 0) tmem_alloc(&S.tmem_slot, P.tmem_cols);
     for (int m = tid; m < P.pd.M; m += MK_THREADS) {
         const int b = P.pd.b0 + m / P.pd.R, pos = P.L[b] + m % P.pd.R, pg = pos / PAGE;
-        s_rowpos[m] = pos < P.rope_rows ? pos : -1;
-        s_rowkv[m] = pg < P.kv.pages_per_seq ? (P.kv.page_table[b * P.kv.pages_per_seq + pg] << 4) | (pos % PAGE) : -1;
+        S.rowpos[m] = pos < P.rope_rows ? pos : -1;
+        S.rowkv[m] = pg < P.kv.pages_per_seq ? (P.kv.page_table[b * P.kv.pages_per_seq + pg] << 4) | (pos % PAGE) : -1;
     }
     // zero the padding rows of the activation tile once (rows >= M are never written)
     for (int q = tid; q < (P.b_dbl ? MAX_ATOMS : HALF_ATOMS) * P.bn * 8; q += MK_THREADS) {
@@ -1050,276 +1369,13 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    const uint32_t tmem = tmem_slot;
-
+    const uint32_t tmem = S.tmem_slot;
     if (warp == 0) {
-        // ---------------- weight producer
-        if (lane == 0) {
-            const uint64_t pol = l2_policy_evict_first();
-            uint32_t kt = 0;
-            for (int i = 0; i < n_my && !aborted(P); ++i) {
-                const MKItem it = my[i];
-                if (it.op != MK_LINEAR) continue;
-                const int lin = it.lin;
-                const bool lt = it.a >= P.n_main[lin] / TILE_ROWS;
-                const uint32_t bytes = lt ? (uint32_t)P.lora_rows[lin] * 128u : (uint32_t)TILE_BYTES;
-                const int kts = P.K[lin] / KT;
-                const uint8_t *src = P.wt[lin] + P.wt_stride[lin] * it.layer +
-                                     ((size_t)it.a * kts + (size_t)it.b * P.katoms[lin]) * TILE_BYTES;
-                bool ok = true;
-                for (int j = 0; j < P.katoms[lin]; ++j, ++kt) {
-                    const int slot = kt % P.nslot;
-                    if (kt >= (uint32_t)P.nslot &&
-                        !mbar_wait_mk(&empty[slot], ((kt / P.nslot) - 1) & 1, P, DEV_TIMEOUT_SLOT)) {
-                        ok = false;
-                        break;
-                    }
-                    mbar_arrive_expect_tx(&full[slot], bytes);
-                    bulk_g2s(ring + (size_t)slot * TILE_BYTES, src + (size_t)j * TILE_BYTES, bytes, &full[slot], pol);
-                }
-                if (!ok) break;
-            }
-            if (aborted(P))  // the last nslot tiles issued may still be in flight: let them land
-                for (uint32_t h = kt > (uint32_t)P.nslot ? kt - P.nslot : 0; h < kt; ++h)
-                    drain_wait(&full[h % P.nslot], (h / P.nslot) & 1);
-        }
+        if (lane == 0) run_producer(P, my, n_my, ring, S);
     } else if (warp == 1) {
-        // ---------------- MMA issuer
-        if (lane == 0) {
-            const uint32_t idesc = idesc_bf16_f32(128, P.bn);
-            uint32_t kt = 0, li = 0, l8 = 0;
-            for (int i = 0; i < n_my; ++i) {
-                const MKItem it = my[i];
-                if (it.op != MK_LINEAR) continue;
-                const int na = P.katoms[it.lin];
-                if (!mbar_wait_mk(&b_full[0], li & 1, P, DEV_TIMEOUT_LOAD)) break;
-                tc_fence_after();
-                bool ok = true;
-                for (int j = 0; j < na; ++j, ++kt) {
-                    if (j == HALF_ATOMS) {
-                        // second half of a wide slice: its operand is staged after the first
-                        // half's reads completed (same area) or was staged with it
-                        if (!P.b_dbl) mma_commit(&b_empty);
-                        if (!mbar_wait_mk(&b_full[1], l8 & 1, P, DEV_TIMEOUT_LOAD)) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
-                    }
-                    const int slot = kt % P.nslot;
-                    if (!mbar_wait_mk(&full[slot], (kt / P.nslot) & 1, P, DEV_TIMEOUT_LOAD)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    const uint64_t ad = sw128_kmajor_desc(ring + (size_t)slot * TILE_BYTES);
-                    const int bj = (P.b_dbl || j < HALF_ATOMS) ? j : j - HALF_ATOMS;
-                    const uint64_t bd = sw128_kmajor_desc(uni + (size_t)bj * P.bn * 128);
-#pragma unroll
-                    for (int kk = 0; kk < KT / 16; ++kk)
-                        mma_bf16_ss(tmem, ad + 2ull * kk, bd + 2ull * kk, idesc, (j | kk) != 0 ? 1u : 0u);
-                    mma_commit(&empty[slot]);
-                }
-                if (!ok) break;
-                mma_commit(&acc_full);
-                ++li;
-                if (na > HALF_ATOMS) ++l8;
-            }
-            if (aborted(P)) {
-                // every MMA issued so far completes before TMEM and the operands are released
-                mma_commit(&mma_drain);
-                drain_wait(&mma_drain, 0);
-            }
-        }
+        if (lane == 0) run_mma(P, my, n_my, ring, uni, tmem, S);
     } else {
-        // ---------------- compute group (warps 2-7)
-        const int ct = tid - 64, cw = warp - 2;
-        uint32_t li = 0, ai = 0, l8 = 0;
-        unsigned long long *tr = P.trace ? P.trace + (size_t)MK_STAMPS * P.cta_off[blockIdx.x] : nullptr;
-        // the attention pages are requested by thread CT_PAGES while thread 0 polls the item's
-        // inputs; att_pend (that thread only): pages requested for a split that has not waited
-        bool att_pend = false;
-        for (int i = 0; i < n_my; ++i) {
-            const MKItem it = my[i];
-            if (tr && ct == 0) {
-                const unsigned long long now = globaltimer_ns();
-                if (i > 0) tr[MK_STAMPS * (i - 1) + 3] = now;
-                tr[MK_STAMPS * i] = now;
-            }
-            const bool att_active = it.op == MK_ATTN && it.c * ATT_SPLIT < P.L[P.pd.b0 + it.a] + P.pd.R;
-            if (att_active && ct == CT_PAGES) {
-                // pages below the cached length do not depend on this pass: fetch them now (the
-                // barrier after the input wait orders this before the split's arrival)
-                attn_pages(P, it.layer, it.a, it.b, it.c, 0, uni, &att_bar, s_phys[0]);
-                att_pend = true;
-            }
-            if (ct == 0) s_flag = wait_deps(P, it) ? 1 : 0;
-            bar_compute();
-            if (!s_flag) break;
-            if (tr && ct == 0) tr[MK_STAMPS * i + 1] = tr[MK_STAMPS * i + 2] = globaltimer_ns();
-            if (it.op == MK_EMBED) {
-                do_embed(P, it.a, cw, lane);
-                bar_compute();
-                if (ct == 0) release_item(P, it);
-            } else if (it.op == MK_FINAL) {
-                const int r = it.a, m = it.b;
-                if (ct == 0) s_rms[0] = row_rms(P, m);
-                bar_compute();
-                const float rs = s_rms[0];
-                for (int c8 = ct; c8 < P.dm.H / 8; c8 += CT) {
-                    const uint4 hv = __ldcg(reinterpret_cast<const uint4 *>(P.h + (size_t)m * P.dm.H) + c8);
-                    const uint4 gv = __ldg(reinterpret_cast<const uint4 *>(P.final_norm) + c8);
-                    const bf16 *he = reinterpret_cast<const bf16 *>(&hv);
-                    const bf16 *ge = reinterpret_cast<const bf16 *>(&gv);
-                    uint4 o;
-                    bf16 *oe = reinterpret_cast<bf16 *>(&o);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) oe[e] = f2bf(__fmul_rn(bf2f(ge[e]), rbf(__fmul_rn(bf2f(he[e]), rs))));
-                    reinterpret_cast<uint4 *>(P.x_ro + (size_t)r * P.dm.H)[c8] = o;
-                }
-            } else if (it.op == MK_ATTN) {
-                const int bl = it.a, g = it.b, s = it.c;
-                if (att_active) {
-                    if (ct == 0) {
-                        attn_pages(P, it.layer, bl, g, s, 1, uni, &att_bar, s_phys[1]);
-                        if (tr) tr[MK_STAMPS * i + 8] = globaltimer_ns();
-                    }
-                    unsigned long long *st = tr ? tr + MK_STAMPS * i : nullptr;
-                    attn_split<DH, DRAFT>(P, it.layer, bl, g, s, uni, &att_bar, ai & 1, ct, cw, lane, st);
-                    ++ai;
-                    att_pend = false;
-                }
-                bar_compute();
-                if (tr && ct == 0) tr[MK_STAMPS * i + 2] = globaltimer_ns();
-                // merge: when the (sequence, head)'s splits fit on distinct CTAs, every split waits for
-                // the others and merges pairs s, s + nsplit, ...; otherwise the last one merges all
-                int *c = ctr(P, it.layer, P.cl.att + bl * P.dm.Hkv + g);
-                const int nsp = P.nsplit[bl];
-                const bool shared_merge = att_shared_merge(nsp);
-                if (ct == 0) {
-                    if (shared_merge) {
-                        red_release_add(c, 1);
-                        s_ok = spin_until(c, nsp, P) ? 1 : 0;
-                        s_red = 1;
-                    } else {
-                        s_red = (atom_acq_rel_add(c, 1) == nsp - 1) ? 1 : 0;
-                        s_ok = 1;
-                    }
-                }
-                if (tr && ct == 0) tr[MK_STAMPS * i + 6] = tr[MK_STAMPS * i + 7] = globaltimer_ns();
-                bar_compute();
-                if (!s_ok) break;
-                if (s_red) {
-                    const int p0 = shared_merge ? s : 0, pstep = shared_merge ? nsp : 1;
-                    attn_combine<DH>(P, bl, g, cw, lane, p0, pstep, tr ? tr + MK_STAMPS * i : nullptr);
-                    bar_compute();
-                    if (ct == 0) release_item(P, it);  // counts on the o slice that reads the group
-                    if (tr && ct == 0) tr[MK_STAMPS * i + 7] = globaltimer_ns();
-                }
-            } else {
-                // ---- linear slice item: stage activations, MMA (warp 1), epilogue, split reduction
-                const int lin = it.lin, l = it.layer, t = it.a, s = it.b;
-                const int na = P.katoms[lin];
-                unsigned long long *st_i = tr ? tr + MK_STAMPS * i : nullptr;
-                if (na <= HALF_ATOMS) {
-                    if (lin == 3)
-                        build_b_act(P, s, uni, ct, s_tag + l, st_i);
-                    else
-                        build_b(P, lin, l, s, uni, s_rms, ct, 0, true, st_i);
-                    fence_proxy_async();
-                    bar_compute();
-                    if (ct == 0) mbarrier_arrive_one(&b_full[0]);
-                } else if (P.b_dbl) {
-                    // wide slice, both halves fit: the first half's MMAs run while the second is staged
-                    build_b(P, lin, l, s, uni, s_rms, ct, 0, true, st_i);
-                    fence_proxy_async();
-                    bar_compute();
-                    if (ct == 0) mbarrier_arrive_one(&b_full[0]);
-                    build_b(P, lin, l, s, uni + (size_t)HALF_ATOMS * P.bn * 128, s_rms, ct, HALF_ATOMS, false,
-                            nullptr);
-                    fence_proxy_async();
-                    bar_compute();
-                    if (ct == 0) mbarrier_arrive_one(&b_full[1]);
-                } else {
-                    // operand in two rounds through the same area
-                    build_b(P, lin, l, s, uni, s_rms, ct, 0, true, st_i);
-                    fence_proxy_async();
-                    bar_compute();
-                    if (ct == 0) {
-                        mbarrier_arrive_one(&b_full[0]);
-                        s_ok = mbar_wait_mk(&b_empty, l8 & 1, P, DEV_TIMEOUT_MMA) ? 1 : 0;
-                    }
-                    bar_compute();
-                    if (!s_ok) break;
-                    build_b(P, lin, l, s, uni, s_rms, ct, HALF_ATOMS, false, nullptr);
-                    fence_proxy_async();
-                    bar_compute();
-                    if (ct == 0) mbarrier_arrive_one(&b_full[1]);
-                }
-                if (na > HALF_ATOMS) ++l8;
-                if (tr && ct == 0) tr[MK_STAMPS * i + 4] = globaltimer_ns();
-                const bool lt = t >= P.n_main[lin] / TILE_ROWS;
-                const int rows_valid = lt ? P.lora_rows[lin] : TILE_ROWS;
-                if (warp >= 4) {
-                    const int quarter = warp - 4;
-                    const bool have = mbar_wait_mk(&acc_full, li & 1, P, DEV_TIMEOUT_MMA);
-                    if (tr && warp == 4 && lane == 0) tr[MK_STAMPS * i + 5] = globaltimer_ns();
-                    tc_fence_after();
-                    if (have) {
-                        const int row = quarter * 32 + lane;
-                        const int n_total = P.n_main[lin] + P.lora_rows[lin];
-                        for (int c0 = 0; c0 < P.bn && c0 < P.pd.M; c0 += 32) {
-                            uint32_t v[32];
-                            tmem_ld_32cols(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)c0, v);
-                            tmem_ld_wait();
-                            if (row < rows_valid) {
-                                unsigned long long *dst =
-                                    P.part[lin] + ((size_t)s * P.part_rows + c0) * n_total + t * TILE_ROWS + row;
-                                const unsigned long long tg = (unsigned long long)(s_tag + l) << 32;
-#pragma unroll
-                                for (int j = 0; j < 32; ++j)
-                                    if (c0 + j < P.pd.M) st_relaxed_u64(dst + (size_t)j * n_total, tg | v[j]);
-                            }
-                        }
-                    }
-                    tc_fence_before();
-                }
-                ++li;
-                bar_compute();
-                if (tr && ct == 0) tr[MK_STAMPS * i + 2] = globaltimer_ns();
-                // The tile's slices are consecutive items of the round-robin schedule, so they sit on
-                // distinct CTAs that all reach them: each CTA stores its tagged slice partials, then
-                // reduces rows s, s + ks, ... of the tile (s = its slice), reading the other slices'
-                // partials as they arrive. The adapter tile's partials are summed by the main tiles'
-                // reducers themselves.
-                const int ks = P.ks[lin];
-                if (tr && ct == 0) tr[MK_STAMPS * i + 6] = globaltimer_ns();
-                if (lt) {
-                    if (tr && ct == 0) tr[MK_STAMPS * i + 7] = globaltimer_ns();
-                    continue;
-                }
-                const uint32_t tag = s_tag + l;
-                if (lin == 0) {
-                    reduce_qkv<DH, DRAFT>(P, l, t, cw, lane, s, ks, tag, s_rowpos, s_rowkv, st_i);
-                } else if (lin == 2)
-                    reduce_gu<DRAFT>(P, l, t, cw, lane, s, ks, tag, st_i);
-                else
-                    reduce_residual<DRAFT>(P, lin, l, t, cw, lane, s, ks, tag, st_i);
-                bar_compute();
-                // one release per reduction, on the counters its consumers poll
-                if (ct == 0) release_item(P, it);
-                if (tr && ct == 0) tr[MK_STAMPS * i + 7] = globaltimer_ns();
-            }
-        }
-        if (tr && ct == 0 && n_my > 0) tr[MK_STAMPS * (n_my - 1) + 3] = globaltimer_ns();
-        if (ct == CT_PAGES && att_pend) {
-            // the pass ended before the split waited for its pages: complete the phase's arrival
-            // and let the copies land (bounded) before the shared memory is released
-            mbarrier_arrive_one(&att_bar);
-            const uint64_t t0 = globaltimer_ns();
-            while (!mbar_try_wait(smem_u32(&att_bar), ai & 1) && globaltimer_ns() - t0 < WAIT_LIMIT_NS) {
-            }
-        }
+        run_compute<DRAFT, DH>(P, my, n_my, uni, tmem, S, tid);
     }
     tc_fence_before();
     __syncthreads();
@@ -1329,7 +1385,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) k_pass(const __grid_constant__ 
         const uint64_t t0 = globaltimer_ns();
         while (ld_relaxed(P.cnt + MK_STARTED) < (int)gridDim.x && globaltimer_ns() - t0 < WAIT_LIMIT_NS) {
         }
-        asm volatile("st.relaxed.gpu.global.b32 [%0], %1;" ::"l"(P.epoch), "r"((int)(s_tag + P.dm.nl - 1)) : "memory");
+        asm volatile("st.relaxed.gpu.global.b32 [%0], %1;" ::"l"(P.epoch), "r"((int)(S.tag + P.dm.nl - 1)) : "memory");
     }
 }
 
