@@ -126,6 +126,7 @@ struct MKParams {
     float *o_part;
     float2 *ml_part;
     int att_splits_alloc;
+    int att_subs;              // partial results per split (1 or 2)
     float att_scale;           // 1/sqrt(head_dim)
     int *status, *abort;
     unsigned long long *trace;  // optional: MK_STAMPS timestamps per item (see pbd_internal.h)
@@ -739,7 +740,7 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
                                         uint64_t *bar, uint32_t parity, int ct, int cw, int lane,
                                         unsigned long long *stamp) {
     constexpr int KS = DH / 16, DT = DH / 8, SUBS = DH / 64;
-    constexpr int HALF = ATT_SPLIT / ATT_SUBS;
+    const int subs = P.att_subs, HALF = ATT_SPLIT / subs;
     const Dims &dm = P.dm;
     const int b = P.pd.b0 + bl;
     const int L = P.L[b];
@@ -782,8 +783,8 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
     const int gq = lane >> 2, tq = lane & 3;
     const float scale = P.att_scale;
 #pragma unroll 1
-    for (int unit = cw; unit < n_mt * ATT_SUBS; unit += CT / 32) {
-        const int mt = unit / ATT_SUBS, half = unit % ATT_SUBS, kb = half * HALF;
+    for (int unit = cw; unit < n_mt * subs; unit += CT / 32) {
+        const int mt = unit / subs, half = unit % subs, kb = half * HALF;
         const int qv0 = mt * 16 + gq, qv1 = qv0 + 8;
         const bool val0 = qv0 < QV, val1 = qv1 < QV;
         const int i0 = val0 ? qv0 / grp : 0, i1 = val1 ? qv1 / grp : 0;
@@ -895,7 +896,7 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
         l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
         l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
         const int nsa = P.att_splits_alloc;
-        const int sub = s * ATT_SUBS + half;  // index of this partial result
+        const int sub = s * subs + half;  // index of this partial result
         if (val0) {
             float *dst = P.o_part + (((size_t)(bl * R + i0) * dm.Hq + h0) * nsa + sub) * DH + 2 * tq;
 #pragma unroll
@@ -921,8 +922,8 @@ __device__ __noinline__ void attn_combine(const MKParams &P, int bl, int g, int 
     const int b = P.pd.b0 + bl;
     const int T = P.L[b] + R;
     const int nsa = P.att_splits_alloc;
-    // partial results computed in this pass: ATT_SUBS per split that holds a key
-    const int nv = min(P.nsplit[bl], (T + ATT_SPLIT - 1) / ATT_SPLIT) * ATT_SUBS;
+    // partial results computed in this pass: att_subs per split that holds a key
+    const int nv = min(P.nsplit[bl], (T + ATT_SPLIT - 1) / ATT_SPLIT) * P.att_subs;
     constexpr int E = DH / 32;
     for (int it = p0 + cw * pstep; it < R * grp; it += (CT / 32) * pstep) {
         const int i = it / grp, h = g * grp + it % grp;
@@ -1596,6 +1597,8 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
     P.o_part = L.o_part;
     P.ml_part = L.ml_part;
     P.att_splits_alloc = L.att_splits_alloc;
+    P.att_subs = L.att_subs;
+    if (L.att_subs < 1 || L.att_subs > ATT_SUBS_MAX) return cudaErrorInvalidValue;
     P.att_scale = (float)(1.0 / std::sqrt((double)L.dm.d));
     P.status = L.status;
     P.trace = L.trace;

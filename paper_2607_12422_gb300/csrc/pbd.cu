@@ -285,8 +285,8 @@ size_t layout(pbd_ctx *c, void *base) {
                              (lin_main(k, lin) + lin_lora(k, lin));
         c->part[lin] = (unsigned long long *)bp.take(c->part_bytes[lin]);
     }
-    c->o_part = (float *)bp.take(sizeof(float) * (size_t)RA * Hq * c->n_splits * ATT_SUBS * d);
-    c->ml_part = (float2 *)bp.take(sizeof(float2) * (size_t)RA * Hq * c->n_splits * ATT_SUBS);
+    c->o_part = (float *)bp.take(sizeof(float) * (size_t)RA * Hq * c->n_splits * ATT_SUBS_MAX * d);
+    c->ml_part = (float2 *)bp.take(sizeof(float2) * (size_t)RA * Hq * c->n_splits * ATT_SUBS_MAX);
     c->tile_max = (float *)bp.take(sizeof(float) * (size_t)(V / TILE_ROWS) * c->ro_alloc);
     c->tile_arg = (int *)bp.take(sizeof(int) * (size_t)(V / TILE_ROWS) * c->ro_alloc);
     c->trace = (unsigned long long *)bp.take(sizeof(unsigned long long) * MK_STAMPS * c->items_cap);
@@ -428,6 +428,14 @@ pbd_status upload_schedule(pbd_ctx *c, int kind, const PassDesc &pd, const std::
     return PBD_OK;
 }
 
+// Partial results per attention split, a constant of the context (every pass of every generation
+// uses the same key partition, so verify rows stay bitwise equal to decode rows): two 64-key halves
+// on separate warps when a full-length pass's split items fit one wave of CTAs; otherwise one warp
+// per query tile over all 128 keys, which halves the partials the merge reads.
+int att_subs_of(const pbd_ctx *c) {
+    return (long)c->cfg.max_batch * c->n_splits * c->cfg.n_kv_heads > c->grid ? 1 : ATT_SUBS_MAX;
+}
+
 MKLaunch make_launch(pbd_ctx *c, const PassDesc &pd, int kind) {
     MKLaunch L;
     const pbd_config &k = c->cfg;
@@ -476,7 +484,8 @@ MKLaunch make_launch(pbd_ctx *c, const PassDesc &pd, int kind) {
     L.ss = c->ss;
     L.o_part = c->o_part;
     L.ml_part = c->ml_part;
-    L.att_splits_alloc = c->n_splits * ATT_SUBS;  // partial results per (row, head)
+    L.att_subs = att_subs_of(c);
+    L.att_splits_alloc = c->n_splits * L.att_subs;  // partial results per (row, head)
     L.status = c->status;
     L.abort = c->cnt;
     return L;

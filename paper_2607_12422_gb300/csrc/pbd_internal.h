@@ -14,7 +14,7 @@ namespace pbd {
 
 constexpr int PAGE = 16;           // KV page length in tokens
 constexpr int ATT_SPLIT = 128;     // key positions per attention split (position-aligned)
-constexpr int ATT_SUBS = 2;        // partial results per split (its two 64-key halves)
+constexpr int ATT_SUBS_MAX = 2;    // partial results per split at most (its two 64-key halves)
 constexpr int PREFILL_ROWS = 64;   // rows per prefill chunk
 constexpr int KT = 64;             // K elements per 128-byte swizzle atom row (bf16)
 constexpr int TILE_ROWS = 128;     // output features per tensor-core tile
@@ -132,6 +132,7 @@ struct MKLaunch {
     float *o_part;
     float2 *ml_part;
     int att_splits_alloc;
+    int att_subs;  // partial results per split: 2 (64-key halves) or 1 (one warp covers the 128 keys)
     int *status, *abort;
     unsigned long long *trace = nullptr;  // optional per-item timestamps
 };
