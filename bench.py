@@ -32,9 +32,11 @@ if ROOT not in sys.path:
 WORKLOAD = "qwen3-0.6b-b1-d16-p512-g256"
 METRIC = "decoded tokens/s (PEFT-BD draft+verify rounds, Qwen3-0.6B shape, D=16)"
 CHUNK = 32  # rounds per timed chunk
-# draft variants measured beside the method of Section 3: early exit at half and quarter depth
-# (Section 6), two-step denoising and the unanchored readout (Sections 4.4 and 5.3)
+# draft variants measured beside the method of Section 3: early exit at half and quarter depth and
+# layer skipping (the odd layers 5..23, 10 of 28; Section 6), two-step denoising and the
+# unanchored readout (Sections 4.4 and 5.3)
 VARIANTS = (("early_exit_14", dict(draft_layers=14)), ("early_exit_7", dict(draft_layers=7)),
+            ("skip_odd_5_23", dict(draft_skip=sum(1 << l for l in range(5, 24, 2)))),
             ("denoise_2", dict(denoise_steps=2)), ("unanchored", dict(anchored=False)))
 
 

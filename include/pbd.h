@@ -69,6 +69,11 @@ typedef struct {
     int32_t draft_unanchored; /* 1: mask row j proposes its own position L+j (rows 1..D are read, the
                                  pending token's row is context only; the unanchored ablation of
                                  Sections 4.4 and 5.3); 0: row j-1 proposes position L+j */
+    uint64_t draft_skip_mask; /* layer skipping (Section 6): bit l set = the draft skips decoder
+                                 layer l (its residual stream passes the layer unchanged and it
+                                 writes no K/V there); 0 = none.  Bits at or above n_layers must be
+                                 clear, and the draft must keep at least one layer (together with
+                                 draft_layers) */
 } pbd_config;
 
 /* Backbone weights: bf16, row-major [out, in] per linear, stacked over layers.  They are

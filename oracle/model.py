@@ -76,7 +76,7 @@ def lib(variant: str = "f32"):
         L.orc_cache_read.argtypes = [C.POINTER(_Config), C.c_void_p, C.c_int32, C.c_int32, C.c_int32, F]
         L.orc_cache_write.argtypes = [C.POINTER(_Config), C.c_void_p, C.c_int32, C.c_int32, C.c_int32, F, F]
         L.orc_forward.argtypes = [C.POINTER(_Config), C.POINTER(_Weights), C.c_void_p, C.c_int32, C.c_int32, I32,
-                                  C.c_int32, C.c_int32, C.c_int32, C.c_int32, F, I32, F]
+                                  C.c_int32, C.c_int32, C.c_int32, C.c_int32, F, I32, F, C.c_uint64]
         L.orc_forward.restype = C.c_int32
         L.orc_op_rmsnorm.argtypes = [C.c_int32, C.c_int32, F, _U16P, C.c_float, F]
         L.orc_op_linear.argtypes = [C.POINTER(_Config), C.c_int32, C.c_int32, C.c_int32, F, _U16P, _U16P, _U16P,
@@ -181,11 +181,13 @@ class OracleModel:
 
     def forward(self, cache: OracleCache, L: int, tokens: Sequence[int], adapter_on: bool, mask_mode: int,
                 read_first: int = 0, n_read: Optional[int] = None, want_logits: bool = False,
-                want_hidden: bool = False, n_layers: Optional[int] = None):
+                want_hidden: bool = False, n_layers: Optional[int] = None, skip_layers: int = 0):
         """One pass over len(tokens) rows at positions L.. (token < 0 = mask row).
 
         n_layers: run only the first n_layers decoder layers, then the final norm and the tied
         head (the early exit of Section 6); the skipped layers' cache slots are left untouched.
+        skip_layers: bit l set skips decoder layer l (layer skipping, Section 6); its cache slots
+        are left untouched too.
         Returns (argmax[n_read], logits[n_read, V] or None, hidden[n_read, H] or None).
         """
         cfg = self.cfg
@@ -204,7 +206,7 @@ class OracleModel:
         rc = lib(self.acc).orc_forward(C.byref(cfg), C.byref(self.weights), cache.ptr, L, n, _i32(toks),
                                int(adapter_on), mask_mode, read_first, n_read,
                                _fp(logits) if logits is not None else None, _i32(am),
-                               _fp(hidden) if hidden is not None else None)
+                               _fp(hidden) if hidden is not None else None, int(skip_layers))
         if rc != 0:
             raise ValueError("oracle forward rejected its arguments (cache capacity or token range)")
         return am, logits, hidden
@@ -233,7 +235,7 @@ def accept_length(draft: Sequence[int], verify: Sequence[int]) -> int:
 
 
 def draft_block(model: OracleModel, cache: OracleCache, L: int, p: int, D: int, draft_layers: Optional[int] = None,
-                denoise_steps: int = 1, anchored: bool = True, want_logits: bool = False):
+                denoise_steps: int = 1, anchored: bool = True, want_logits: bool = False, draft_skip: int = 0):
     """The adapter-on draft of one round (Section 3, steps 1-2) and its variants.
 
     Step 1 runs rows [p, MASK x D] at positions L..L+D under the block mask.  The token it
@@ -245,7 +247,8 @@ def draft_block(model: OracleModel, cache: OracleCache, L: int, p: int, D: int, 
     runs the same adapter-on block pass with the mask rows replaced by the previous step's
     proposals, rows [p, d_1..d_D], nothing remasked; its proposals replace the block.
     draft_layers: the draft exits after the first draft_layers decoder layers (the early exit
-    Section 6 names as a cheaper draft path); None runs all of them.
+    Section 6 names as a cheaper draft path); None runs all of them.  draft_skip: a mask of
+    decoder layers the draft skips (layer skipping, the other cheaper path Section 6 names).
     Returns (drafts of the last step, its logits or None, proposals of every step).
     """
     first = 0 if anchored else 1
@@ -254,7 +257,7 @@ def draft_block(model: OracleModel, cache: OracleCache, L: int, p: int, D: int, 
     lg = None
     for _ in range(max(1, denoise_steps)):
         am, lg, _ = model.forward(cache, L, rows, True, MASK_BLOCK_DRAFT, first, D, want_logits=want_logits,
-                                  n_layers=draft_layers)
+                                  n_layers=draft_layers, skip_layers=draft_skip)
         drafts = [int(t) for t in am]
         steps.append(drafts)
         rows = [p] + drafts
@@ -278,14 +281,15 @@ def spec_generate(model: OracleModel, prompt: Sequence[int], max_new: int, D: in
                   forced_n: Optional[Sequence[int]] = None,
                   draft_override: Optional[Callable[[int, List[int]], List[int]]] = None,
                   want_logits: bool = False, max_rounds: Optional[int] = None, return_state: bool = False,
-                  draft_layers: Optional[int] = None, denoise_steps: int = 1, anchored: bool = True):
+                  draft_layers: Optional[int] = None, denoise_steps: int = 1, anchored: bool = True,
+                  draft_skip: int = 0):
     """PEFT-BD decoding (Section 3).  Returns (tokens, rounds[, (cache, L)]).
 
     rounds[i] = dict(L=cached length before the round, pending, draft, verify, n, emitted,
     draft_steps, [draft_logits, verify_logits]).  forced_n replaces the accepted length of
     round i by forced_n[i] (timing mode); draft_override(i, drafts) may replace the drafted
-    block (adversarial drafters in the tests).  draft_layers, denoise_steps and anchored
-    select the draft variant (draft_block).  The generation budget is the only stop rule:
+    block (adversarial drafters in the tests).  draft_layers, denoise_steps, anchored and
+    draft_skip select the draft variant (draft_block).  The generation budget is the only stop rule:
     the last round is truncated to max_new tokens.
     """
     P = len(prompt)
@@ -296,7 +300,7 @@ def spec_generate(model: OracleModel, prompt: Sequence[int], max_new: int, D: in
     while len(out) < max_new and (max_rounds is None or len(rounds) < max_rounds):
         ri = len(rounds)
         drafts, d_lg, d_steps = draft_block(model, cache, L, p, D, draft_layers, denoise_steps, anchored,
-                                            want_logits)
+                                            want_logits, draft_skip)
         if draft_override is not None:
             drafts = [int(t) for t in draft_override(ri, list(drafts))]
         v_am, v_lg, _ = model.forward(cache, L, [p] + drafts, False, MASK_CAUSAL, 0, D + 1,

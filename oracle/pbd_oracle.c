@@ -310,7 +310,7 @@ int orc_cache_read(const orc_config *c, const orc_cache *cc, int32_t layer, int3
  * Returns 0, or 1 when the cache is too small. */
 int orc_forward(const orc_config *c, const orc_weights *w, orc_cache *cache, int32_t L, int32_t n,
                 const int32_t *tokens, int32_t adapter_on, int32_t mask_mode, int32_t read_first, int32_t n_read,
-                float *logits, int32_t *argmax, float *hidden_out) {
+                float *logits, int32_t *argmax, float *hidden_out, uint64_t skip_layers) {
     if (L < 0 || n <= 0 || L + n > cache->capacity) return 1;
     if (read_first < 0 || read_first + n_read > n) return 1;
     for (int i = 0; i < n; i++)
@@ -334,6 +334,10 @@ int orc_forward(const orc_config *c, const orc_weights *w, orc_cache *cache, int
     }
 
     for (int l = 0; l < c->n_layers; l++) {
+        /* layer skipping (Section 6 names it beside the early exit as a cheaper draft path):
+         * a layer whose bit is set in skip_layers leaves the residual stream untouched and
+         * writes no K/V */
+        if (l < 64 && ((skip_layers >> l) & 1u)) continue;
         const uint16_t *Wl[N_LIN], *Al[N_LIN], *Bl[N_LIN];
         for (int t = 0; t < N_LIN; t++) {
             int fin, fout;

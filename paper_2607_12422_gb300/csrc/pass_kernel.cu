@@ -1423,8 +1423,8 @@ void mk_counter_layout(const Dims &dm, int max_nb, CounterLayout *cl) {
 // i, i+grid, ...), so each CTA's list is in dependency order.  Returns items sorted by CTA.
 // Every item carries the one counter it waits for and the counters it adds to once done:
 //   embed row       -> embed counter (target M for layer 0's q|k|v)
-//   q|k|v slice     waits for layer l-1's residual after down (8 tiles x 12 slices at 0.6B) or the
-//                   embeddings; its reduction counts on att_in of each KV group its tile feeds
+//   q|k|v slice     waits for the previous layer run's residual after down (8 tiles x 12 slices at
+//                   0.6B) or the embeddings; its reduction counts on att_in of each KV group it feeds
 //   attention split waits for att_in of its group (every slice of every q, k, v tile of the
 //                   group); the (sequence, group) merge counter orders the split's own merge, and a
 //                   finished merge counts on att_o of the o slice that reads the group
@@ -1482,7 +1482,9 @@ void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int
     for (int bl = 0; bl < pd.nb; ++bl) merges += nsplit[bl] <= grid ? nsplit[bl] : 1;
     const int o_w = mk_slice_atoms(1, K[1]) * KT;  // o slice width
     for (int m = 0; m < pd.M; ++m) push(MK_EMBED, 0, 0, m, 0, 0, -1, 0, cl.embed, -1);
+    int prev = -1;  // the last layer run so far (skipped layers have no items)
     for (int l = 0; l < pd.nl_run; ++l) {
+        if (l < 64 && ((pd.skip >> l) & 1u)) continue;
         auto linear = [&](int lin, int wait_off, int wait_tgt) {
             for (int r = 0; r < (pd.adapter ? 1 : 0) + n_main[lin]; ++r) {
                 const int t = pd.adapter ? (r == 0 ? n_main[lin] : r - 1) : r;  // adapter tile first
@@ -1502,10 +1504,11 @@ void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int
                 for (int sl = 0; sl < ks[lin]; ++sl) push(MK_LINEAR, lin, l, t, sl, 0, wait_off, wait_tgt, rel0, rel1);
             }
         };
-        if (l == 0)
+        if (prev < 0)
             linear(0, cl.embed, pd.M);
         else
-            linear(0, ctr(l - 1, cl.res_dn), n_main[3] * ks[3]);
+            linear(0, ctr(prev, cl.res_dn), n_main[3] * ks[3]);
+        prev = l;
         for (int bl = 0; bl < pd.nb; ++bl)
             for (int g = 0; g < dm.Hkv; ++g)
                 for (int sp = 0; sp < nsplit[bl]; ++sp)
@@ -1526,8 +1529,8 @@ void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int
     }
     for (int bl = 0; bl < pd.nb; ++bl)
         for (int i = pd.ro_first; i < pd.ro_first + pd.ro_count; ++i)
-            push(MK_FINAL, 0, pd.nl_run - 1, bl * pd.ro_count + (i - pd.ro_first), bl * pd.R + i, 0,
-                 ctr(pd.nl_run - 1, cl.res_dn), n_main[3] * ks[3], -1, -1);
+            push(MK_FINAL, 0, prev, bl * pd.ro_count + (i - pd.ro_first), bl * pd.R + i, 0, ctr(prev, cl.res_dn),
+                 n_main[3] * ks[3], -1, -1);
     off->assign(grid + 1, 0);
     for (size_t i = 0; i < all.size(); ++i) (*off)[i % grid + 1]++;
     for (int c = 0; c < grid; ++c) (*off)[c + 1] += (*off)[c];

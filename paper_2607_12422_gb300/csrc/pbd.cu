@@ -179,6 +179,14 @@ bool valid_config(const pbd_config *cfg, std::string *why) {
     if (k.draft_layers < 0 || k.draft_layers > k.n_layers) return bad("draft_layers must be in [0, n_layers]");
     if (k.denoise_steps < 0 || k.denoise_steps > 8) return bad("denoise_steps must be in [0, 8]");
     if (k.draft_unanchored != 0 && k.draft_unanchored != 1) return bad("draft_unanchored must be 0 or 1");
+    if (k.n_layers < 64 && (k.draft_skip_mask >> k.n_layers) != 0)
+        return bad("draft_skip_mask has bits at or above n_layers");
+    {
+        const int E = k.draft_layers > 0 ? k.draft_layers : k.n_layers;
+        int kept = 0;
+        for (int l = 0; l < E; ++l) kept += (l < 64 && ((k.draft_skip_mask >> l) & 1u)) ? 0 : 1;
+        if (kept == 0) return bad("the draft must keep at least one layer");
+    }
     return true;
 }
 
@@ -407,6 +415,7 @@ PassDesc block_pass(pbd_ctx *c, int kind) {
     pd.ro_first = (kind == PK_DRAFT && c->cfg.draft_unanchored) ? 1 : 0;
     pd.ro_count = kind == PK_DRAFT ? c->D : pd.R;
     pd.nl_run = draft_pass_layers(c, kind);
+    pd.skip = kind == PK_DRAFT ? c->cfg.draft_skip_mask : 0;
     return pd;
 }
 
@@ -580,7 +589,9 @@ double pass_bytes(pbd_ctx *c, int kind, const std::vector<int> &Ls) {
         w += 2.0 * lin_main(k, lin) * lin_K(k, lin);
         lora += 2.0 * k.lora_rank * (lin_K(k, lin) + lin_main(k, lin));
     }
-    const int nl = draft_pass_layers(c, kind);
+    int nl = 0;  // decoder layers the pass runs
+    for (int l = 0; l < draft_pass_layers(c, kind); ++l)
+        nl += (kind == PK_DRAFT && l < 64 && ((k.draft_skip_mask >> l) & 1u)) ? 0 : 1;
     double bytes = nl * (w + (kind == PK_DRAFT ? lora : 0.0));
     bytes += 2.0 * (2.0 * nl * k.hidden + 2.0 * nl * k.head_dim);  // norm gains
     const double kv_tok = 2.0 * 2.0 * nl * k.n_kv_heads * k.head_dim;

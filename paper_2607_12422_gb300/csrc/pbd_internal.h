@@ -35,6 +35,7 @@ struct PassDesc {
     int ro_first;    // read-out rows per sequence: i in [ro_first, ro_first + ro_count)
     int ro_count;
     int nl_run;      // decoder layers the pass runs before the final norm (the draft's early exit)
+    uint64_t skip = 0;  // decoder layers below nl_run the pass skips (the draft's layer skipping)
 };
 
 // Paged KV cache: [layer][page][Hkv][PAGE][d] bf16 for K and for V.

@@ -36,7 +36,8 @@ class pbd_config(C.Structure):
                 ("vocab", C.c_int32), ("rms_eps", C.c_float), ("rope_theta", C.c_float),
                 ("lora_rank", C.c_int32), ("lora_scale", C.c_float), ("block_D", C.c_int32),
                 ("max_batch", C.c_int32), ("max_seq_len", C.c_int32), ("page_size", C.c_int32),
-                ("draft_layers", C.c_int32), ("denoise_steps", C.c_int32), ("draft_unanchored", C.c_int32)]
+                ("draft_layers", C.c_int32), ("denoise_steps", C.c_int32), ("draft_unanchored", C.c_int32),
+                ("draft_skip_mask", C.c_uint64)]
 
 
 class pbd_base_weights(C.Structure):
@@ -215,12 +216,12 @@ def pbd_op_lm_head_argmax(x, E, want_logits: bool = False):
 
 
 def make_config(shape, block_D: int, max_batch: int, max_seq_len: int, draft_layers: int = 0,
-                denoise_steps: int = 1, anchored: bool = True) -> pbd_config:
+                denoise_steps: int = 1, anchored: bool = True, draft_skip: int = 0) -> pbd_config:
     """pbd_config for a model shape; the draft variant defaults to the method of Section 3."""
     return pbd_config(shape.n_layers, shape.hidden, shape.n_q_heads, shape.n_kv_heads, shape.head_dim,
                       shape.intermediate, shape.vocab, shape.rms_eps, shape.rope_theta, shape.lora_rank,
                       shape.lora_alpha / shape.lora_rank, block_D, max_batch, max_seq_len, 16,
-                      draft_layers, denoise_steps, 0 if anchored else 1)
+                      draft_layers, denoise_steps, 0 if anchored else 1, draft_skip)
 
 
 def pbd_plan_pass(cfg: pbd_config, kind: int, prompt_lens: Sequence[int], max_new: int, grid: int,
@@ -248,14 +249,15 @@ class Engine:
 
     def __init__(self, shape, base: Dict[str, np.ndarray], adapter: Dict[str, np.ndarray], block_D: int,
                  max_batch: int, max_seq_len: int, device: str = "cuda:0", keep_host_weights: bool = False,
-                 draft_layers: int = 0, denoise_steps: int = 1, anchored: bool = True):
+                 draft_layers: int = 0, denoise_steps: int = 1, anchored: bool = True, draft_skip: int = 0):
         import torch
         self.torch = torch
         self.lib = load()
         self.shape = shape
         self.D = block_D
         self.device = torch.device(device)
-        self.cfg = make_config(shape, block_D, max_batch, max_seq_len, draft_layers, denoise_steps, anchored)
+        self.cfg = make_config(shape, block_D, max_batch, max_seq_len, draft_layers, denoise_steps, anchored,
+                               draft_skip)
         need = self.lib.pbd_workspace_bytes(C.byref(self.cfg))
         if need == 0:
             raise PbdError(1, "configuration rejected by pbd_workspace_bytes")

@@ -1,12 +1,12 @@
 """Parity of the draft variants on the GPU against the CPU oracle: the early exit after E
-decoder layers (Section 6), two-step denoising and the unanchored readout (Sections 4.4
-and 5.3).
+decoder layers and layer skipping (Section 6), two-step denoising and the unanchored readout
+(Sections 4.4 and 5.3).
 
 Tiny model (2 layers, D = 16): rounds in lockstep with the oracle (draft logits within
 3e-2, draft ids equal up to ties inside that tolerance, verify logits and ids likewise,
 accepted lengths, cached lengths and pending tokens exact), then the whole generation
-equal to greedy decoding.  Qwen3-0.6B shape: the half-depth early-exit draft in lockstep
-for one round (tolerance derived as in the full-depth lockstep test), and every variant's
+equal to greedy decoding.  Qwen3-0.6B shape: the half-depth early-exit draft and a draft
+skipping the odd layers 5..23 in lockstep for one round (tolerance derived as in the full-depth lockstep test), and every variant's
 speculative output equal to plain greedy decoding on the same kernels, bit for bit."""
 import numpy as np
 import pytest
@@ -20,6 +20,7 @@ D = 16
 
 VARIANTS = [
     dict(draft_layers=1),
+    dict(draft_skip=1),
     dict(denoise_steps=2),
     dict(anchored=False),
     dict(draft_layers=1, denoise_steps=2, anchored=False),
@@ -32,7 +33,7 @@ def _ident(v):
 
 def _oracle_kw(var):
     return dict(draft_layers=var.get("draft_layers"), denoise_steps=var.get("denoise_steps", 1),
-                anchored=var.get("anchored", True))
+                anchored=var.get("anchored", True), draft_skip=var.get("draft_skip", 0))
 
 
 def _check_ids(ids, ref_logits, tol=TOL):
@@ -125,9 +126,10 @@ def test_variant_generate_is_greedy(tenv, var):
 
 def test_variant_config_rejected(tenv):
     pbd = tenv["pbd"]
-    with pytest.raises(pbd.PbdError):
-        pbd.Engine(tenv["S"], tenv["base"], tenv["ad"], block_D=D, max_batch=1, max_seq_len=256,
-                   draft_layers=tenv["S"].n_layers + 1)
+    for kw in (dict(draft_layers=tenv["S"].n_layers + 1), dict(draft_skip=3), dict(draft_skip=4),
+               dict(draft_layers=1, draft_skip=1)):
+        with pytest.raises(pbd.PbdError):
+            pbd.Engine(tenv["S"], tenv["base"], tenv["ad"], block_D=D, max_batch=1, max_seq_len=256, **kw)
 
 
 @pytest.fixture(scope="module")
@@ -143,12 +145,17 @@ def qenv():
     return dict(torch=torch, pbd=pbd, S=S, base=base, ad=ad, prompt=prompt)
 
 
-def test_qwen_half_depth_draft_lockstep(qenv):
+SKIP_ODD_5_23 = sum(1 << l for l in range(5, 24, 2))
+
+
+@pytest.mark.parametrize("var", [dict(draft_layers=14), dict(draft_skip=SKIP_ODD_5_23)], ids=["exit14", "skip-odd-5-23"])
+def test_qwen_cheaper_draft_lockstep(qenv, var):
     pbd, S, prompt = qenv["pbd"], qenv["S"], qenv["prompt"]
-    E = S.n_layers // 2
+    E = var.get("draft_layers")
+    skip = var.get("draft_skip", 0)
     m = oracle.OracleModel(S, qenv["base"], qenv["ad"])
     m64 = oracle.OracleModel(S, qenv["base"], qenv["ad"], acc="f64acc")
-    eng = pbd.Engine(S, qenv["base"], qenv["ad"], block_D=D, max_batch=1, max_seq_len=1024, draft_layers=E)
+    eng = pbd.Engine(S, qenv["base"], qenv["ad"], block_D=D, max_batch=1, max_seq_len=1024, **var)
     P = len(prompt)
     first = eng.pbd_prefill([prompt], max_new=64)
     cache, p, lg0 = m.prefill(prompt, P + 2 * (D + 1), want_logits=True)
@@ -156,8 +163,8 @@ def test_qwen_half_depth_draft_lockstep(qenv):
     if int(first[0]) != p:
         _check_ids([int(first[0])], lg0[None])
         pytest.skip("first token is a near-tie between GPU and oracle; lockstep needs a common start")
-    od_ids, od, _ = oracle.draft_block(m, cache, P, p, D, draft_layers=E, want_logits=True)
-    _, od64, _ = oracle.draft_block(m64, cache64, P, p, D, draft_layers=E, want_logits=True)
+    od_ids, od, _ = oracle.draft_block(m, cache, P, p, D, draft_layers=E, want_logits=True, draft_skip=skip)
+    _, od64, _ = oracle.draft_block(m64, cache64, P, p, D, draft_layers=E, want_logits=True, draft_skip=skip)
     tol = min(0.1, max(TOL, 2 * float(np.abs(od - od64).max())))
     d_ids, d_lg = eng.pbd_draft_block(want_logits=True)
     assert np.abs(d_lg[0].cpu().numpy() - od).max() <= tol
@@ -165,7 +172,8 @@ def test_qwen_half_depth_draft_lockstep(qenv):
     eng.close()
 
 
-@pytest.mark.parametrize("var", [dict(draft_layers=14), dict(denoise_steps=2), dict(anchored=False)], ids=_ident)
+@pytest.mark.parametrize("var", [dict(draft_layers=14), dict(denoise_steps=2), dict(anchored=False),
+                                 dict(draft_skip=SKIP_ODD_5_23)], ids=_ident)
 def test_qwen_variant_spec_equals_ar_bitwise(qenv, var):
     pbd, S, prompt = qenv["pbd"], qenv["S"], qenv["prompt"]
     eng = pbd.Engine(S, qenv["base"], qenv["ad"], block_D=D, max_batch=1, max_seq_len=1024, **var)

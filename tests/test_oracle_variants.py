@@ -3,6 +3,9 @@
 - Early exit after E decoder layers (a cheaper draft path, Section 6): the draft's logits
   equal those of a separately built model holding only the first E layers' weights, and
   E = n_layers is the default draft bit for bit.
+- Layer skipping (the other cheaper draft path Section 6 names): the draft with a set of
+  layers skipped equals a separately built model holding only the kept layers' weights, fed
+  the kept layers' cache; an empty skip set is the default draft bit for bit.
 - Unanchored readout (Sections 4.4 and 5.3): the same block pass read one row later, so
   the unanchored proposals d_1..d_{D-1} are the anchored proposals d_2..d_D.
 - Two-step denoising (Sections 4.4 and 5.3): step 1 is the one-step draft; the pending
@@ -21,6 +24,7 @@ from oracle import MASK_CAUSAL
 
 VARIANTS = [
     dict(draft_layers=1),
+    dict(draft_skip=1),
     dict(denoise_steps=2),
     dict(anchored=False),
     dict(draft_layers=1, denoise_steps=2, anchored=False),
@@ -67,6 +71,42 @@ def test_early_exit_equals_truncated_model(tiny):
     assert not np.array_equal(lg_full, lg_ee)
 
 
+def _kept_model(tiny, keep):
+    """The same backbone and adapter holding only the decoder layers in `keep`, in order."""
+    S = tiny["shape"]
+    S2 = dataclasses.replace(S, n_layers=len(keep))
+    per_layer = ("attn_norm", "mlp_norm", "q_norm", "k_norm") + tuple("w" + n for n in oracle.LINEAR_NAMES)
+    base = {k: (np.ascontiguousarray(v[keep]) if k in per_layer else v) for k, v in tiny["base"].items()}
+    ad = {k: (np.ascontiguousarray(v[keep]) if k != "mask_embed" else v) for k, v in tiny["adapter"].items()}
+    return oracle.OracleModel(S2, base, ad)
+
+
+def test_layer_skip_equals_model_of_kept_layers(tiny):
+    """Skipping layer 0 of the two: the draft equals a one-layer model holding layer 1's weights,
+    with layer 1's cache of the prefix; a wrong layer (the skipped one's weights) differs."""
+    m, prompt, S = tiny["model"], tiny["prompt"], tiny["shape"]
+    P, D = len(prompt), 8
+    assert S.n_layers == 2
+    cache, p, _ = m.prefill(prompt, P + 32)
+    d_sk, lg_sk, _ = oracle.draft_block(m, cache, P, p, D, draft_skip=1, want_logits=True)
+    for keep, same in (([1], True), ([0], False)):
+        kept = _kept_model(tiny, keep)
+        c2 = kept.new_cache(P + 32)
+        c2.write(0, 0, cache.read(keep[0], "k", P), cache.read(keep[0], "v", P))
+        d2, lg2, _ = oracle.draft_block(kept, c2, P, p, D, want_logits=True)
+        assert np.array_equal(lg_sk.view(np.uint32), lg2.view(np.uint32)) == same, keep
+        if same:
+            assert d_sk == d2
+    # an empty skip set is the default draft
+    d0, l0, _ = oracle.draft_block(m, cache, P, p, D, want_logits=True)
+    d1, l1, _ = oracle.draft_block(m, cache, P, p, D, draft_skip=0, want_logits=True)
+    assert d0 == d1 and np.array_equal(l0.view(np.uint32), l1.view(np.uint32))
+    # the skipped layer's cache slots are not written by the draft
+    before = cache.read(0, "k", P + D + 1).copy()
+    oracle.draft_block(m, cache, P, p, D, draft_skip=1)
+    assert np.array_equal(cache.read(0, "k", P + D + 1)[P:], before[P:])
+
+
 def test_early_exit_at_depth_is_default_draft(tiny):
     m, prompt = tiny["model"], tiny["prompt"]
     P, D = len(prompt), 8
@@ -107,7 +147,7 @@ def test_variant_rounds_commit_prefill_kv(tiny):
     m, prompt, S = tiny["model"], tiny["prompt"], tiny["shape"]
     D = 4
     out, rounds, (cache, L) = oracle.spec_generate(m, prompt, 40, D, return_state=True, draft_layers=1,
-                                                   denoise_steps=2, anchored=False)
+                                                   denoise_steps=2, anchored=False, draft_skip=1)
     toks = list(prompt) + out[:-1]
     assert L == len(toks)
     fresh = m.new_cache(L + 8)

@@ -258,3 +258,24 @@ def test_check_catches_planted_mistakes(mistake):
         bad = np.concatenate([bad[:i], bad[i + 1:j + 1], bad[i:i + 1], bad[j + 1:]])
     with pytest.raises(AssertionError):
         _check(S, *_redeal(bad, grid), grid, S.n_layers, [256, 256, 256, 256])
+
+
+def test_layer_skip_schedule():
+    """A draft skipping layers: no item of a skipped layer, each kept layer's q|k|v waits for the
+    previous kept layer's residual, the final norm for the last kept layer; counters consistent."""
+    S = synth.QWEN3_0_6B
+    skip = sum(1 << l for l in range(5, 24, 2))
+    cfg = pbd.make_config(S, 16, 1, 1024, draft_skip=skip)
+    items, off = pbd.pbd_plan_pass(cfg, 0, [512], 256, 152)
+    _check_counters(items, off, 152)
+    op, lin, layer, a, b, c = _decode(items)
+    kept = [l for l in range(S.n_layers) if not (skip >> l) & 1]
+    assert set(layer[op == OP_LINEAR]) == set(kept)
+    assert set(layer[op == OP_FINAL]) == {kept[-1]}
+    # the verify pass of the same context runs every layer
+    items_v, off_v = pbd.pbd_plan_pass(cfg, 1, [512], 256, 152)
+    _check(S, items_v, off_v, 152, S.n_layers, [256, 256, 512, 256])
+    # a mask keeping no layer, or naming a layer beyond the model, is rejected
+    for bad in ((1 << S.n_layers) - 1, 1 << S.n_layers):
+        with pytest.raises(pbd.PbdError):
+            pbd.pbd_plan_pass(pbd.make_config(S, 16, 1, 1024, draft_skip=bad), 0, [512], 256, 152)
