@@ -50,7 +50,7 @@ constexpr int HALF_ATOMS = 4;      // 64-wide swizzle atoms of one operand stagi
 constexpr int MAX_ATOMS = 8;       // atoms per linear item at most (K slice 512)
 constexpr int MAX_SLOT = 12;
 constexpr int MK_STARTED = 1;      // global counter slot: CTAs that have read the pass counter
-constexpr int CT_PAGES = 32;       // compute thread (warp 3, lane 0) that requests attention pages
+constexpr int CT_PAGES = 32;       // first compute thread of the warp (warp 3) that requests attention pages
 constexpr int RING_SLOTS = 4;      // weight tiles in the ring (64 KiB)
 constexpr int MAX_ROWS = 256;
 
@@ -683,49 +683,45 @@ __device__ __forceinline__ uint32_t sw128(int row, int colb) {
     return (uint32_t)(row * 128 + ((((colb >> 4) ^ (row & 7)) << 4) | (colb & 15)));
 }
 
-// TMA loads of the pages of one attention split, issued by one thread of the compute group.
-// stage 0: pages entirely below the cached length L (written by earlier passes: prefetched
-// before the item's inputs are ready); stage 1: pages holding this pass's block rows.  Announces
-// the stage's bytes on `bar` (stage 1 with the item's one arrival) before issuing the copies.
-// The page-table entries are read together first (one round trip), kept in `phys` (8 shared ints
-// owned by the calling thread).  Returns the stage's bytes.
-__device__ __noinline__ uint32_t attn_pages(const MKParams &P, int layer, int bl, int g, int s, int stage,
-                                            uint8_t *smem, uint64_t *bar, int *phys) {
+// TMA loads of the pages of one attention split, issued by one warp of the compute group (all
+// lanes call): stage 0 = pages entirely below the cached length L (written by earlier passes:
+// requested before the item's inputs are ready); stage 1 = pages holding this pass's block rows.
+// Lane p < 8 reads the page-table entry of page p (one round trip for all); lane 0 announces the
+// stage's bytes on `bar` (stage 1 with the item's one arrival); then every lane issues one of the
+// split's copies (page l / (2 subs), K or V, 64-dim half), so the warp issues them together.
+__device__ __noinline__ void attn_pages(const MKParams &P, int layer, int bl, int g, int s, int stage, uint8_t *smem,
+                                        uint64_t *bar, int lane) {
     constexpr int NP = ATT_SPLIT / PAGE;
     const int b = P.pd.b0 + bl;
     const int L = P.L[b], T = L + P.pd.R, k0 = s * ATT_SPLIT, pg0 = k0 / PAGE;
-    const int *pt = P.kv.page_table + (size_t)b * P.kv.pages_per_seq + pg0;
-    unsigned mask = 0;
-    int ph[NP];
-#pragma unroll
-    for (int p = 0; p < NP; ++p) {
-        const int kp0 = k0 + p * PAGE;
-        const bool ok = kp0 < T && pg0 + p < P.kv.pages_per_seq && ((kp0 + PAGE <= L) == (stage == 0));
-        mask |= (ok ? 1u : 0u) << p;
-        ph[p] = ok ? pt[p] : 0;
+    int ph = 0;
+    bool ok = false;
+    if (lane < NP) {
+        const int kp0 = k0 + lane * PAGE;
+        ok = kp0 < T && pg0 + lane < P.kv.pages_per_seq && ((kp0 + PAGE <= L) == (stage == 0));
+        if (ok) ph = P.kv.page_table[(size_t)b * P.kv.pages_per_seq + pg0 + lane];
     }
-#pragma unroll
-    for (int p = 0; p < NP; ++p) phys[p] = ph[p];
-    const int subs = P.dm.d / 64;
-    const uint32_t bytes = (uint32_t)__popc(mask) * (uint32_t)subs * 2u * PAGE * 128u;
-    // the block's pages were written by this pass's q|k|v reducers (generic stores, acquired
-    // before this call): order them before the TMA reads
-    if (stage == 1 && mask) fence_proxy_async_global();
-    if (stage == 1)
-        mbar_arrive_expect_tx(bar, bytes);
-    else if (bytes)
-        mbar_expect_tx(bar, bytes);
-#pragma unroll 1
-    for (int p = 0; p < NP; ++p) {
-        if (!((mask >> p) & 1u)) continue;
-        const int row0 = ((layer * P.kv.n_pages + phys[p]) * P.dm.Hkv + g) * PAGE;
-#pragma unroll 1
-        for (int sub = 0; sub < subs; ++sub) {
-            tma_load_2d(smem + sub * ATT_SUB_BYTES + p * PAGE * 128, &P.kmap, sub * 64, row0, bar);
-            tma_load_2d(smem + (subs + sub) * ATT_SUB_BYTES + p * PAGE * 128, &P.vmap, sub * 64, row0, bar);
-        }
+    const unsigned mask = __ballot_sync(0xffffffffu, ok);
+    const int subs = P.dm.d / 64, tpp = 2 * subs;  // copies per page: K and V, per 64-dim half
+    if (lane == 0) {
+        const uint32_t bytes = (uint32_t)__popc(mask) * (uint32_t)tpp * PAGE * 128u;
+        if (stage == 1)
+            mbar_arrive_expect_tx(bar, bytes);
+        else if (bytes)
+            mbar_expect_tx(bar, bytes);
     }
-    return bytes;
+    __syncwarp();
+    const int p = lane / tpp, r = lane % tpp;
+    const int phys = __shfl_sync(0xffffffffu, ph, p < NP ? p : 0);
+    if (p < NP && ((mask >> p) & 1u)) {
+        // the block's pages were written by this pass's q|k|v reducers (generic stores, acquired
+        // before this call): order them before the TMA reads
+        if (stage == 1) fence_proxy_async_global();
+        const int kind = r / subs, sub = r % subs;
+        const int row0 = ((layer * P.kv.n_pages + phys) * P.dm.Hkv + g) * PAGE;
+        tma_load_2d(smem + (kind * subs + sub) * ATT_SUB_BYTES + p * PAGE * 128, kind ? &P.vmap : &P.kmap, sub * 64,
+                    row0, bar);
+    }
 }
 
 // One (sequence, KV head, 128-key split) on the compute group, after its K/V pages landed in
@@ -1007,7 +1003,6 @@ struct CtaState {
     int flag, red, ok;
     uint32_t tag;  // this pass's partial-sum tag
     float rms[MAX_ROWS];
-    int phys[2][ATT_SPLIT / PAGE];  // page ids of attention stages 0 and 1
     // per pass row: position (-1 beyond the RoPE table) and KV slot (page << 4 | slot; -1 beyond
     // the reserved pages)
     int rowpos[MAX_ROWS], rowkv[MAX_ROWS];
@@ -1127,9 +1122,9 @@ __device__ __noinline__ bool item_attn(const MKParams &P, const MKItem &it, bool
                                        uint32_t &ai, int ct, int cw, int lane, unsigned long long *st) {
     const int bl = it.a, g = it.b, s = it.c;
     if (active) {
-        if (ct == 0) {
-            attn_pages(P, it.layer, bl, g, s, 1, uni, &S.att_bar, S.phys[1]);
-            stamp_at(st, 8);
+        if (cw == 0) {
+            attn_pages(P, it.layer, bl, g, s, 1, uni, &S.att_bar, lane);
+            if (lane == 0) stamp_at(st, 8);
         }
         attn_split<DH, DRAFT>(P, it.layer, bl, g, s, uni, &S.att_bar, ai & 1, ct, cw, lane, st);
         ++ai;
@@ -1268,7 +1263,7 @@ __device__ __noinline__ bool item_linear(const MKParams &P, const MKItem &it, ui
 }
 
 // ---- compute group (warps 2-7): dependency waits, operand staging, epilogues, reductions,
-// attention; the attention's cached pages are requested by thread CT_PAGES while thread 0 polls
+// attention; the attention's cached pages are requested by warp CT_PAGES / 32 while thread 0 polls
 // the item's inputs
 template <bool DRAFT, int DH>
 __device__ __noinline__ void run_compute(const MKParams &P, const MKItem *my, int n_my, uint8_t *uni, uint32_t tmem,
@@ -1276,7 +1271,7 @@ __device__ __noinline__ void run_compute(const MKParams &P, const MKItem *my, in
     const int ct = tid - 64, cw = ct >> 5, lane = tid & 31, warp = tid >> 5;
     uint32_t li = 0, ai = 0, l8 = 0;
     unsigned long long *tr = P.trace ? P.trace + (size_t)MK_STAMPS * P.cta_off[blockIdx.x] : nullptr;
-    bool att_pend = false;  // (thread CT_PAGES) pages requested for a split that has not waited
+    bool att_pend = false;  // (that warp) pages requested for a split that has not waited
 #pragma unroll 1
     for (int i = 0; i < n_my; ++i) {
         const MKItem it = my[i];
@@ -1287,10 +1282,10 @@ __device__ __noinline__ void run_compute(const MKParams &P, const MKItem *my, in
             st[0] = now;
         }
         const bool att_active = it.op == MK_ATTN && it.c * ATT_SPLIT < P.L[P.pd.b0 + it.a] + P.pd.R;
-        if (att_active && ct == CT_PAGES) {
+        if (att_active && cw == CT_PAGES / 32) {
             // pages below the cached length do not depend on this pass: fetch them now (the
             // barrier after the input wait orders this before the split's arrival)
-            attn_pages(P, it.layer, it.a, it.b, it.c, 0, uni, &S.att_bar, S.phys[0]);
+            attn_pages(P, it.layer, it.a, it.b, it.c, 0, uni, &S.att_bar, lane);
             att_pend = true;
         }
         if (ct == 0) S.flag = wait_deps(P, it) ? 1 : 0;
