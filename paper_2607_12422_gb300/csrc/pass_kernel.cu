@@ -727,7 +727,7 @@ __device__ __noinline__ void attn_pages(const MKParams &P, int layer, int bl, in
 // One (sequence, KV head, 128-key split) on the compute group, after its K/V pages landed in
 // `smem` (stages 0 and 1 of attn_pages) and `bar` completed phase `parity`.  Each warp takes one
 // 16-row query tile and one 64-key half of the split; the halves are separate partial results
-// (m, l, O) that the merge combines like splits.  Within a half the keys go in chunks of 16 with
+// (m, l, O) that the merge combines like splits.  Within a half the keys go in chunks of 32 with
 // a running maximum (online softmax): scores by bf16 mma.sync, the row maximum and the weights in
 // fp32, P (weights) in fp16 against V converted to fp16, O in fp32.  The loop over chunks is not
 // unrolled: the code stays small enough for the instruction cache.
@@ -747,29 +747,25 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
     const int QV = R * grp;
     const int n_mt = (QV + 15) / 16;
     uint8_t *sK = smem, *sV = smem + SUBS * ATT_SUB_BYTES;
-    // pages without keys of this pass were not loaded: zero their V rows (p = 0 there, and
-    // 0 * stale bits could be NaN); their K rows are masked
-    const int kv_end = min(T, P.kv.pages_per_seq * PAGE);  // keys at or past this were not loaded
-    if (k0 + ATT_SPLIT > kv_end) {
-        const int row0 = max(0, (kv_end - k0 + PAGE - 1) / PAGE * PAGE);
-#pragma unroll 1
-        for (int idx = row0 * 8 * SUBS + ct; idx < ATT_SPLIT * 8 * SUBS; idx += CT) {
-            const int sub = idx & (SUBS - 1), rc = idx / SUBS;  // (row, chunk) = rc / 8, rc % 8
-            *reinterpret_cast<uint4 *>(sV + sub * ATT_SUB_BYTES + (rc >> 3) * 128 + (rc & 7) * 16) = make_uint4(0, 0, 0, 0);
-        }
-    }
     const bool landed = mbar_wait_mk(bar, parity, P, DEV_TIMEOUT_LOAD);
     if (stamp && ct == 0) stamp[4] = globaltimer_ns();
-    // V to fp16 in place (each 16-byte chunk independently; the swizzle layout is unchanged)
+    // V to fp16 in place (each 16-byte chunk independently; the swizzle layout is unchanged).
+    // Rows of keys at or past T become zeros: their weights are 0, but their slots hold whatever
+    // the cache held (a page's tail beyond the sequence, or pages not loaded at all), and 0 times
+    // an Inf or NaN there would poison the sum.  Their K rows are masked out of the scores.
 #pragma unroll 1
     for (int idx = ct; idx < SUBS * ATT_SUB_BYTES / 16; idx += CT) {
         uint4 *p4 = reinterpret_cast<uint4 *>(sV + idx * 16);
-        uint4 v4 = *p4;
-        uint32_t *w = reinterpret_cast<uint32_t *>(&v4);
+        const int key = (idx % (ATT_SUB_BYTES / 16)) >> 3;  // 8 chunks of 16 bytes per key row
+        uint4 v4 = make_uint4(0, 0, 0, 0);
+        if (k0 + key < T) {
+            v4 = *p4;
+            uint32_t *w = reinterpret_cast<uint32_t *>(&v4);
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[e]));
-            w[e] = pack_half2(f.x, f.y);
+            for (int e = 0; e < 4; ++e) {
+                const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[e]));
+                w[e] = pack_half2(f.x, f.y);
+            }
         }
         *p4 = v4;
     }
@@ -807,11 +803,12 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
 #pragma unroll
         for (int dt = 0; dt < DT; ++dt) oc[dt][0] = oc[dt][1] = oc[dt][2] = oc[dt][3] = 0.f;
         const int kend = min(HALF, T - (k0 + kb));  // keys of the half that exist
+        constexpr int CN = 4;  // n-tiles of 8 keys per chunk (32 keys)
 #pragma unroll 1
-        for (int c0 = 0; c0 < kend; c0 += 16) {
-            float sc[2][4];
+        for (int c0 = 0; c0 < kend; c0 += 8 * CN) {
+            float sc[CN][4];
 #pragma unroll
-            for (int nt = 0; nt < 2; ++nt) {
+            for (int nt = 0; nt < CN; ++nt) {
                 sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
                 // K fragments of two k-steps per ldmatrix.x4: matrix j = keys n0..n0+7, dims 8j..8j+7
                 // of the 32-dim chunk; thread t addresses row t % 8 of matrix t / 8
@@ -830,7 +827,7 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
             }
             float c0m = -INFINITY, c1m = -INFINITY;
 #pragma unroll
-            for (int nt = 0; nt < 2; ++nt)
+            for (int nt = 0; nt < CN; ++nt)
 #pragma unroll
                 for (int e = 0; e < 2; ++e) {
                     const int kp = k0 + kb + c0 + nt * 8 + 2 * tq + e;
@@ -844,22 +841,25 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
             c1m = fmaxf(c1m, __shfl_xor_sync(0xffffffffu, c1m, 1));
             c1m = fmaxf(c1m, __shfl_xor_sync(0xffffffffu, c1m, 2));
             const float n0 = fmaxf(m0, c0m), n1 = fmaxf(m1, c1m);
-            // rescale what was summed so far to the new maximum (nothing was, while it is -inf)
-            const float a0 = m0 == -INFINITY ? 0.f : __expf(m0 - n0), a1 = m1 == -INFINITY ? 0.f : __expf(m1 - n1);
+            // rescale what was summed so far to the new maximum (nothing was while it is -inf;
+            // skipped by the whole warp when no row's maximum moved)
+            if (__any_sync(0xffffffffu, (n0 != m0 && m0 != -INFINITY) || (n1 != m1 && m1 != -INFINITY))) {
+                const float a0 = m0 == -INFINITY ? 0.f : __expf(m0 - n0), a1 = m1 == -INFINITY ? 0.f : __expf(m1 - n1);
+                l0 = __fmul_rn(l0, a0);
+                l1 = __fmul_rn(l1, a1);
+#pragma unroll
+                for (int dt = 0; dt < DT; ++dt) {
+                    oc[dt][0] = __fmul_rn(oc[dt][0], a0);
+                    oc[dt][1] = __fmul_rn(oc[dt][1], a0);
+                    oc[dt][2] = __fmul_rn(oc[dt][2], a1);
+                    oc[dt][3] = __fmul_rn(oc[dt][3], a1);
+                }
+            }
             const float z0 = n0 == -INFINITY ? 0.f : n0, z1 = n1 == -INFINITY ? 0.f : n1;
             m0 = n0;
             m1 = n1;
-            l0 = __fmul_rn(l0, a0);
-            l1 = __fmul_rn(l1, a1);
 #pragma unroll
-            for (int dt = 0; dt < DT; ++dt) {
-                oc[dt][0] = __fmul_rn(oc[dt][0], a0);
-                oc[dt][1] = __fmul_rn(oc[dt][1], a0);
-                oc[dt][2] = __fmul_rn(oc[dt][2], a1);
-                oc[dt][3] = __fmul_rn(oc[dt][3], a1);
-            }
-#pragma unroll
-            for (int nt = 0; nt < 2; ++nt)
+            for (int nt = 0; nt < CN; ++nt)
 #pragma unroll
                 for (int e = 0; e < 2; ++e) {
                     sc[nt][e] = sc[nt][e] == -INFINITY ? 0.f : __expf(sc[nt][e] - z0);
@@ -867,23 +867,26 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
                     l0 += sc[nt][e];
                     l1 += sc[nt][2 + e];
                 }
-            // P as the fp16 A fragment of one 16-key step
-            uint32_t pa[4];
-            pa[0] = pack_half2(sc[0][0], sc[0][1]);
-            pa[1] = pack_half2(sc[0][2], sc[0][3]);
-            pa[2] = pack_half2(sc[1][0], sc[1][1]);
-            pa[3] = pack_half2(sc[1][2], sc[1][3]);
-            const int vrow = kb + c0 + (lane & 7) + ((lane >> 3) & 1) * 8;
+            // P as the fp16 A fragments of two 16-key steps
 #pragma unroll
-            for (int dt = 0; dt < DT; dt += 2) {
-                const int vcol = dt * 8 + (lane >> 4) * 8;
-                const uint32_t addr = smem_u32(sV + (vcol >> 6) * ATT_SUB_BYTES + sw128(vrow, (vcol & 63) * 2));
-                uint32_t r0, r1, r2, r3;
-                asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-                             : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-                             : "r"(addr));
-                mma_m16n8k16_f16(oc[dt], pa, r0, r1);
-                mma_m16n8k16_f16(oc[dt + 1], pa, r2, r3);
+            for (int kstep = 0; kstep < CN / 2; ++kstep) {
+                uint32_t pa[4];
+                pa[0] = pack_half2(sc[2 * kstep][0], sc[2 * kstep][1]);
+                pa[1] = pack_half2(sc[2 * kstep][2], sc[2 * kstep][3]);
+                pa[2] = pack_half2(sc[2 * kstep + 1][0], sc[2 * kstep + 1][1]);
+                pa[3] = pack_half2(sc[2 * kstep + 1][2], sc[2 * kstep + 1][3]);
+                const int vrow = kb + c0 + kstep * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+#pragma unroll
+                for (int dt = 0; dt < DT; dt += 2) {
+                    const int vcol = dt * 8 + (lane >> 4) * 8;
+                    const uint32_t addr = smem_u32(sV + (vcol >> 6) * ATT_SUB_BYTES + sw128(vrow, (vcol & 63) * 2));
+                    uint32_t r0, r1, r2, r3;
+                    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                                 : "r"(addr));
+                    mma_m16n8k16_f16(oc[dt], pa, r0, r1);
+                    mma_m16n8k16_f16(oc[dt + 1], pa, r2, r3);
+                }
             }
         }
         stamp_at(sw, 10);
