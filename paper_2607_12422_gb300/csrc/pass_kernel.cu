@@ -239,16 +239,15 @@ __device__ __forceinline__ float row_rms(const MKParams &P, int m) {
     return __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(__fdiv_rn(a, (float)P.dm.H), P.dm.eps)));
 }
 
-// sum_j u_j * B[f, j] over j = 0..r-1 in order (B row: r bf16 values, r % 8 == 0)
 // one B row (r bf16 values) of the adapter, for lora_dot_w
 struct BRow {
     uint4 w[MAX_RANK / 8];
 };
-__device__ __forceinline__ BRow load_brow(const bf16 *Brow, int r) {
+// the B row of local tile row j, from the tile's B rows staged in shared memory (r / 8 chunks each)
+__device__ __forceinline__ BRow smem_brow(const uint4 *brows, int j, int r) {
     BRow b;
 #pragma unroll
-    for (int q = 0; q < MAX_RANK / 8; ++q)
-        b.w[q] = q * 8 < r ? __ldg(reinterpret_cast<const uint4 *>(Brow) + q) : make_uint4(0, 0, 0, 0);
+    for (int q = 0; q < MAX_RANK / 8; ++q) b.w[q] = q * 8 < r ? brows[j * (r / 8) + q] : make_uint4(0, 0, 0, 0);
     return b;
 }
 __device__ __forceinline__ float lora_dot_w(const float (&u)[MAX_RANK], const BRow &b, int r) {
@@ -491,7 +490,8 @@ __device__ __noinline__ void build_b_act(const MKParams &P, int slice, uint8_t *
 // at kernel start.
 template <int DH, bool AD>
 __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, int cw, int lane, int m0, int mstep,
-                                       uint32_t tag, const int *rowpos, const int *rowkv, unsigned long long *st) {
+                                       uint32_t tag, const int *rowpos, const int *rowkv, const uint4 *brows,
+                                       unsigned long long *st) {
     constexpr int LPH = DH / 4;  // lanes per head
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r;
@@ -501,7 +501,6 @@ __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, 
     const int head = (ft - (kind == 0 ? 0 : (kind == 1 ? qw : qw + kvw))) / DH + hl;
     const int f0 = ft + 4 * lane;
     const bool lo = e0 < DH / 2;  // first half of the head (RoPE: x cos - partner sin)
-    const bf16 *lb = P.lora_b[0] + (size_t)layer * P.lb_stride[0];
     float g[4];
     if (kind < 2) {
         const uint2 graw = __ldg(reinterpret_cast<const uint2 *>((kind == 0 ? P.q_norm : P.k_norm) + (size_t)layer * DH + e0));
@@ -509,10 +508,6 @@ __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, 
         const float2 gb = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&graw.y));
         g[0] = ga.x, g[1] = ga.y, g[2] = gb.x, g[3] = gb.y;
     }
-    BRow br[4];
-    if (AD)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) br[j] = load_brow(lb + (size_t)(f0 + j) * r, r);
 #pragma unroll 1
     for (int m = m0 + cw * mstep; m < M; m += (CT / 32) * mstep) {
         const int pos = rowpos[m];
@@ -531,7 +526,7 @@ __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, 
         if (AD) share_u(y[4], 0, u);
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-            if (AD) y[j] = __fadd_rn(y[j], __fmul_rn(dm.lora_scale, lora_dot_w(u, br[j], r)));
+            if (AD) y[j] = __fadd_rn(y[j], __fmul_rn(dm.lora_scale, lora_dot_w(u, smem_brow(brows, 4 * lane + j, r), r)));
             y[j] = rbf(y[j]);
         }
         if (kind < 2) {
@@ -582,16 +577,10 @@ __device__ __noinline__ void reduce_qkv(const MKParams &P, int layer, int tile, 
 // then across the lanes by a fixed butterfly.
 template <bool AD>
 __device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int layer, int tile, int cw, int lane, int m0,
-                                             int mstep, uint32_t tag, unsigned long long *st) {
+                                             int mstep, uint32_t tag, const uint4 *brows, unsigned long long *st) {
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r, H = dm.H, nt = H / TILE_ROWS;
     const int f0 = tile * TILE_ROWS + 4 * lane;
-    const bf16 *lb = P.lora_b[lin] + (size_t)layer * P.lb_stride[lin];
-    // B rows depend only on the feature: loaded once, before the rows
-    BRow br[4];
-    if (AD)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) br[e] = load_brow(lb + (size_t)(f0 + e) * r, r);
 #pragma unroll 1
     for (int m = m0 + cw * mstep; m < M; m += (CT / 32) * mstep) {
         uint2 *hp = reinterpret_cast<uint2 *>(P.h + (size_t)m * H + f0);
@@ -608,7 +597,7 @@ __device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int lay
         float v[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-            if (AD) acc[e] = __fadd_rn(acc[e], __fmul_rn(dm.lora_scale, lora_dot_w(u, br[e], r)));
+            if (AD) acc[e] = __fadd_rn(acc[e], __fmul_rn(dm.lora_scale, lora_dot_w(u, smem_brow(brows, 4 * lane + e, r), r)));
             v[e] = rbf(__fadd_rn(hv[e], rbf(acc[e])));
         }
         uint2 o;
@@ -631,18 +620,10 @@ __device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int lay
 // 64 + 2l + 1) and stores them as one tagged word.
 template <bool AD>
 __device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, int cw, int lane, int m0, int mstep,
-                                      uint32_t tag, unsigned long long *st) {
+                                      uint32_t tag, const uint4 *brows, unsigned long long *st) {
     const Dims &dm = P.dm;
     const int M = P.pd.M, r = dm.r, I = dm.I;
     const int a0 = tile * 64 + 2 * lane;  // the lane's first act feature
-    const bf16 *lb = P.lora_b[2] + (size_t)layer * P.lb_stride[2];
-    BRow bg[2], bu[2];
-    if (AD)
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-            bg[e] = load_brow(lb + (size_t)(a0 + e) * r, r);
-            bu[e] = load_brow(lb + (size_t)(I + a0 + e) * r, r);
-        }
 #pragma unroll 1
     for (int m = m0 + cw * mstep; m < M; m += (CT / 32) * mstep) {
         // sums: gate pair, up pair; feature 4: adapter row lane (lanes 0..r-1 sum u_gate, r..2r-1 u_up)
@@ -659,8 +640,8 @@ __device__ __noinline__ void reduce_gu(const MKParams &P, int layer, int tile, i
         for (int e = 0; e < 2; ++e) {
             float g = s[e], up = s[2 + e];
             if (AD) {
-                g = __fadd_rn(g, __fmul_rn(dm.lora_scale, lora_dot_w(ug, bg[e], r)));
-                up = __fadd_rn(up, __fmul_rn(dm.lora_scale, lora_dot_w(uu, bu[e], r)));
+                g = __fadd_rn(g, __fmul_rn(dm.lora_scale, lora_dot_w(ug, smem_brow(brows, 2 * lane + e, r), r)));
+                up = __fadd_rn(up, __fmul_rn(dm.lora_scale, lora_dot_w(uu, smem_brow(brows, 64 + 2 * lane + e, r), r)));
             }
             g = rbf(g);
             up = rbf(up);
@@ -1009,6 +990,9 @@ struct CtaState {
     // per pass row: position (-1 beyond the RoPE table) and KV slot (page << 4 | slot; -1 beyond
     // the reserved pages)
     int rowpos[MAX_ROWS], rowkv[MAX_ROWS];
+    // the adapter's B rows of the tile a draft's linear item reduces (tile row order: for
+    // gate|up rows 0-63 gate, 64-127 up), staged at the item's start
+    uint4 brows[TILE_ROWS * MAX_RANK / 8];
 };
 
 // ---- warp 0 lane 0: weight producer.  Walks the CTA's linear items ahead of the others and
@@ -1178,10 +1162,24 @@ __device__ __noinline__ bool item_linear(const MKParams &P, const MKItem &it, ui
                                          unsigned long long *st) {
     const int lin = it.lin, l = it.layer, t = it.a, s = it.b;
     const int na = P.katoms[lin];
+    if (DRAFT && t < P.n_main[lin] / TILE_ROWS) {
+        // the adapter's B rows of this tile: they depend only on (layer, tile), so they are copied
+        // while the operand is staged (the staging's cp.async wait covers them)
+        const int r = P.dm.r, cpr = r / 8;  // 16-byte chunks per B row
+        const bf16 *lb = P.lora_b[lin] + (size_t)l * P.lb_stride[lin];
+#pragma unroll 1
+        for (int q = ct; q < TILE_ROWS * cpr; q += CT) {
+            const int j = q / cpr, c = q % cpr;
+            const int f = lin == 2 ? (j < 64 ? t * 64 + j : P.dm.I + t * 64 + (j - 64)) : t * TILE_ROWS + j;
+            cp_async16(&S.brows[q], lb + (size_t)f * r + c * 8);
+        }
+        cp_async_commit();
+    }
     if (na <= HALF_ATOMS) {
-        if (lin == 3)
+        if (lin == 3) {
             build_b_act(P, s, uni, ct, S.tag + l, st);
-        else
+            if (DRAFT) cp_async_wait_all();  // the B rows (the operand needed no copies)
+        } else
             build_b(P, lin, l, s, uni, S.rms, ct, 0, true, st);
         fence_proxy_async();
         bar_compute();
@@ -1251,11 +1249,11 @@ __device__ __noinline__ bool item_linear(const MKParams &P, const MKItem &it, ui
     }
     const int ks = P.ks[lin];
     if (lin == 0)
-        reduce_qkv<DH, DRAFT>(P, l, t, cw, lane, s, ks, tag, S.rowpos, S.rowkv, st);
+        reduce_qkv<DH, DRAFT>(P, l, t, cw, lane, s, ks, tag, S.rowpos, S.rowkv, S.brows, st);
     else if (lin == 2)
-        reduce_gu<DRAFT>(P, l, t, cw, lane, s, ks, tag, st);
+        reduce_gu<DRAFT>(P, l, t, cw, lane, s, ks, tag, S.brows, st);
     else
-        reduce_residual<DRAFT>(P, lin, l, t, cw, lane, s, ks, tag, st);
+        reduce_residual<DRAFT>(P, lin, l, t, cw, lane, s, ks, tag, S.brows, st);
     bar_compute();
     // one release per reduction, on the counters its consumers poll
     if (ct == 0) {
