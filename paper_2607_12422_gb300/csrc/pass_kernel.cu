@@ -101,7 +101,7 @@ struct MKParams {
     const int *cta_off;
     int *cnt;            // counters of this pass (zeroed before launch)
     CounterLayout cl;
-    const int *nsplit;   // [nb] attention split items per sequence
+    const int *nsplit;   // [nb] 128-key attention splits per sequence (items: ceil(nsplit / att_span))
     // weights
     const uint8_t *wt[4];      // tiled weights of layer 0; layer stride wt_stride[lin] bytes
     size_t wt_stride[4];
@@ -664,20 +664,23 @@ __device__ __forceinline__ uint32_t sw128(int row, int colb) {
     return (uint32_t)(row * 128 + ((((colb >> 4) ^ (row & 7)) << 4) | (colb & 15)));
 }
 
-// TMA loads of the pages of one attention split, issued by one warp of the compute group (all
-// lanes call): stage 0 = pages entirely below the cached length L (written by earlier passes:
-// requested before the item's inputs are ready); stage 1 = pages holding this pass's block rows.
-// Lane p < 8 reads the page-table entry of page p (one round trip for all); lane 0 announces the
-// stage's bytes on `bar` (stage 1 with the item's one arrival); then every lane issues one of the
-// split's copies (page l / (2 subs), K or V, 64-dim half), so the warp issues them together.
+// TMA loads of the pages of one attention item (att_span consecutive 128-key splits), issued by
+// one warp of the compute group (all lanes call): stage 0 = pages entirely below the cached length
+// L (written by earlier passes: requested before the item's inputs are ready); stage 1 = pages
+// holding this pass's block rows.  Lane p < 8 * span reads the page-table entry of the item's page
+// p (one round trip for all); lane 0 announces the stage's bytes on `bar` (stage 1 with the item's
+// one arrival); then the lanes issue the copies (page, K or V, 64-dim half) together, one per lane
+// and round.  Split j of the item lands at smem + j * 2 (d/64) ATT_SUB_BYTES: its K halves, then its
+// V halves.
 __device__ __noinline__ void attn_pages(const MKParams &P, int layer, int bl, int g, int s, int stage, uint8_t *smem,
                                         uint64_t *bar, int lane) {
     constexpr int NP = ATT_SPLIT / PAGE;
+    const int span = P.pd.att_span, npg = NP * span;
     const int b = P.pd.b0 + bl;
-    const int L = P.L[b], T = L + P.pd.R, k0 = s * ATT_SPLIT, pg0 = k0 / PAGE;
+    const int L = P.L[b], T = L + P.pd.R, k0 = s * span * ATT_SPLIT, pg0 = k0 / PAGE;
     int ph = 0;
     bool ok = false;
-    if (lane < NP) {
+    if (lane < npg) {
         const int kp0 = k0 + lane * PAGE;
         ok = kp0 < T && pg0 + lane < P.kv.pages_per_seq && ((kp0 + PAGE <= L) == (stage == 0));
         if (ok) ph = P.kv.page_table[(size_t)b * P.kv.pages_per_seq + pg0 + lane];
@@ -692,54 +695,61 @@ __device__ __noinline__ void attn_pages(const MKParams &P, int layer, int bl, in
             mbar_expect_tx(bar, bytes);
     }
     __syncwarp();
-    const int p = lane / tpp, r = lane % tpp;
-    const int phys = __shfl_sync(0xffffffffu, ph, p < NP ? p : 0);
-    if (p < NP && ((mask >> p) & 1u)) {
-        // the block's pages were written by this pass's q|k|v reducers (generic stores, acquired
-        // before this call): order them before the TMA reads
-        if (stage == 1) fence_proxy_async_global();
-        const int kind = r / subs, sub = r % subs;
-        const int row0 = ((layer * P.kv.n_pages + phys) * P.dm.Hkv + g) * PAGE;
-        tma_load_2d(smem + (kind * subs + sub) * ATT_SUB_BYTES + p * PAGE * 128, kind ? &P.vmap : &P.kmap, sub * 64,
-                    row0, bar);
+    // the block's pages were written by this pass's q|k|v reducers (generic stores, acquired
+    // before this call): order them before the TMA reads
+    if (stage == 1 && mask) fence_proxy_async_global();
+#pragma unroll 1
+    for (int c0 = 0; c0 < npg * tpp; c0 += 32) {  // uniform over the warp: one or two rounds
+        const int cp = c0 + lane, p = min(cp / tpp, 31), r = cp % tpp;
+        const int phys = __shfl_sync(0xffffffffu, ph, p);
+        if (cp < npg * tpp && ((mask >> p) & 1u)) {
+            const int kind = r / subs, sub = r % subs, sp = p / NP;
+            const int row0 = ((layer * P.kv.n_pages + phys) * P.dm.Hkv + g) * PAGE;
+            tma_load_2d(smem + ((sp * 2 + kind) * subs + sub) * ATT_SUB_BYTES + (p % NP) * PAGE * 128,
+                        kind ? &P.vmap : &P.kmap, sub * 64, row0, bar);
+        }
     }
 }
 
-// One (sequence, KV head, 128-key split) on the compute group, after its K/V pages landed in
-// `smem` (stages 0 and 1 of attn_pages) and `bar` completed phase `parity`.  Each warp takes one
-// 16-row query tile and one 64-key half of the split; the halves are separate partial results
-// (m, l, O) that the merge combines like splits.  Within a half the keys go in chunks of 32 with
-// a running maximum (online softmax): scores by bf16 mma.sync, the row maximum and the weights in
-// fp32, P (weights) in fp16 against V converted to fp16, O in fp32.  The loop over chunks is not
-// unrolled: the code stays small enough for the instruction cache.
+// One (sequence, KV head, att_span 128-key splits) item on the compute group, after its K/V pages
+// landed in `smem` (stages 0 and 1 of attn_pages) and `bar` completed phase `parity`.  Each warp
+// takes units of one 16-row query tile against one split's keys, or one 64-key half of them when a
+// split has two partial results; every unit is a partial result (m, l, O) that the merge combines
+// in key order; the partition of the keys does not depend on the span.  Within a unit the keys go
+// in chunks of 32 with a running maximum (online softmax): scores by bf16 mma.sync, the row maximum
+// and the weights in fp32, P (weights) in fp16 against V converted to fp16, O in fp32.  The loop
+// over chunks is not unrolled: the code stays small enough for the instruction cache.
 template <int DH, bool BLK>
 __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, int g, int s, uint8_t *smem,
                                         uint64_t *bar, uint32_t parity, int ct, int cw, int lane,
                                         unsigned long long *stamp) {
     constexpr int KS = DH / 16, DT = DH / 8, SUBS = DH / 64;
+    constexpr int SPB = 2 * SUBS * ATT_SUB_BYTES;  // staged bytes per split (K, then V)
     const int subs = P.att_subs, HALF = ATT_SPLIT / subs;
     const Dims &dm = P.dm;
     const int b = P.pd.b0 + bl;
     const int L = P.L[b];
     const int R = P.pd.R;
     const int T = L + R;
-    const int k0 = s * ATT_SPLIT;
+    const int sp0 = s * P.pd.att_span;  // the item's first split
+    const int nsx = min(P.pd.att_span, (T - sp0 * ATT_SPLIT + ATT_SPLIT - 1) / ATT_SPLIT);  // splits holding keys
     const int grp = dm.Hq / dm.Hkv;
     const int QV = R * grp;
     const int n_mt = (QV + 15) / 16;
-    uint8_t *sK = smem, *sV = smem + SUBS * ATT_SUB_BYTES;
     const bool landed = mbar_wait_mk(bar, parity, P, DEV_TIMEOUT_LOAD);
     if (stamp && ct == 0) stamp[4] = globaltimer_ns();
     // V to fp16 in place (each 16-byte chunk independently; the swizzle layout is unchanged).
     // Rows of keys at or past T become zeros: their weights are 0, but their slots hold whatever
     // the cache held (a page's tail beyond the sequence, or pages not loaded at all), and 0 times
     // an Inf or NaN there would poison the sum.  Their K rows are masked out of the scores.
+    constexpr int VCH = SUBS * ATT_SUB_BYTES / 16;  // 16-byte chunks of one split's V
 #pragma unroll 1
-    for (int idx = ct; idx < SUBS * ATT_SUB_BYTES / 16; idx += CT) {
-        uint4 *p4 = reinterpret_cast<uint4 *>(sV + idx * 16);
-        const int key = (idx % (ATT_SUB_BYTES / 16)) >> 3;  // 8 chunks of 16 bytes per key row
+    for (int idx = ct; idx < nsx * VCH; idx += CT) {
+        const int sp = idx / VCH, w = idx % VCH;
+        uint4 *p4 = reinterpret_cast<uint4 *>(smem + sp * SPB + SUBS * ATT_SUB_BYTES + w * 16);
+        const int key = (w % (ATT_SUB_BYTES / 16)) >> 3;  // 8 chunks of 16 bytes per key row
         uint4 v4 = make_uint4(0, 0, 0, 0);
-        if (k0 + key < T) {
+        if ((sp0 + sp) * ATT_SPLIT + key < T) {
             v4 = *p4;
             uint32_t *w = reinterpret_cast<uint32_t *>(&v4);
 #pragma unroll
@@ -756,8 +766,10 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
     const int gq = lane >> 2, tq = lane & 3;
     const float scale = P.att_scale;
 #pragma unroll 1
-    for (int unit = cw; unit < n_mt * subs; unit += CT / 32) {
-        const int mt = unit / subs, half = unit % subs, kb = half * HALF;
+    for (int unit = cw; unit < n_mt * nsx * subs; unit += CT / 32) {
+        const int mt = unit / (nsx * subs), sp = (unit / subs) % nsx, half = unit % subs, kb = half * HALF;
+        const int k0 = (sp0 + sp) * ATT_SPLIT;
+        const uint8_t *sK = smem + sp * SPB, *sV = sK + SUBS * ATT_SUB_BYTES;
         const int qv0 = mt * 16 + gq, qv1 = qv0 + 8;
         const bool val0 = qv0 < QV, val1 = qv1 < QV;
         const int i0 = val0 ? qv0 / grp : 0, i1 = val1 ? qv1 / grp : 0;
@@ -876,7 +888,7 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
         l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
         l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
         const int nsa = P.att_splits_alloc;
-        const int sub = s * subs + half;  // index of this partial result
+        const int sub = (sp0 + sp) * subs + half;  // index of this partial result
         if (val0) {
             float *dst = P.o_part + (((size_t)(bl * R + i0) * dm.Hq + h0) * nsa + sub) * DH + 2 * tq;
 #pragma unroll
@@ -961,8 +973,8 @@ __device__ __noinline__ void attn_combine(const MKParams &P, int bl, int g, int 
     }
 }
 
-// Attention merge mode of a (sequence, head) with nsp splits: shared by all splits when they sit
-// on distinct CTAs (nsp <= grid), else done by the last split.
+// Attention merge mode of a (sequence, head) with nsp items: shared by all items when they sit on
+// distinct CTAs (nsp <= grid), else done by the last one.
 __device__ __forceinline__ bool att_shared_merge(int nsp) { return nsp <= (int)gridDim.x; }
 
 // the item's inputs are complete (one thread; false on abort)
@@ -1118,10 +1130,10 @@ __device__ __noinline__ bool item_attn(const MKParams &P, const MKItem &it, bool
     }
     bar_compute();
     if (ct == 0) stamp_at(st, 2);
-    // merge: when the (sequence, head)'s splits fit on distinct CTAs, every split waits for the
-    // others and merges pairs s, s + nsplit, ...; otherwise the last one merges all
+    // merge: when the (sequence, head)'s items fit on distinct CTAs, every item waits for the
+    // others and merges pairs s, s + items, ...; otherwise the last one merges all
     int *c = ctr(P, it.layer, P.cl.att + bl * P.dm.Hkv + g);
-    const int nsp = P.nsplit[bl];
+    const int nsp = (P.nsplit[bl] + P.pd.att_span - 1) / P.pd.att_span;
     const bool shared_merge = att_shared_merge(nsp);
     if (ct == 0) {
         if (shared_merge) {
@@ -1282,7 +1294,8 @@ __device__ __noinline__ void run_compute(const MKParams &P, const MKItem *my, in
             if (i > 0) tr[MK_STAMPS * (i - 1) + 3] = now;
             st[0] = now;
         }
-        const bool att_active = it.op == MK_ATTN && it.c * ATT_SPLIT < P.L[P.pd.b0 + it.a] + P.pd.R;
+        const bool att_active =
+            it.op == MK_ATTN && it.c * P.pd.att_span * ATT_SPLIT < P.L[P.pd.b0 + it.a] + P.pd.R;
         if (att_active && cw == CT_PAGES / 32) {
             // pages below the cached length do not depend on this pass: fetch them now (the
             // barrier after the input wait orders this before the split's arrival)
@@ -1473,9 +1486,14 @@ void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int
         tile_groups(t, &g0, &g1);
         for (int g = g0; g <= g1; ++g) att_in_tgt[g] += ks[0];
     }
-    // merges per (sequence, group): every split when the splits sit on distinct CTAs, else the last
+    // attention items per sequence (each covers att_span consecutive 128-key splits) and merges per
+    // (sequence, group): every item when the items sit on distinct CTAs, else the last
+    const int span = pd.att_span;
     int merges = 0;
-    for (int bl = 0; bl < pd.nb; ++bl) merges += nsplit[bl] <= grid ? nsplit[bl] : 1;
+    for (int bl = 0; bl < pd.nb; ++bl) {
+        const int items = (nsplit[bl] + span - 1) / span;
+        merges += items <= grid ? items : 1;
+    }
     const int o_w = mk_slice_atoms(1, K[1]) * KT;  // o slice width
     for (int m = 0; m < pd.M; ++m) push(MK_EMBED, 0, 0, m, 0, 0, -1, 0, cl.embed, -1);
     int prev = -1;  // the last layer run so far (skipped layers have no items)
@@ -1507,7 +1525,7 @@ void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int
         prev = l;
         for (int bl = 0; bl < pd.nb; ++bl)
             for (int g = 0; g < dm.Hkv; ++g)
-                for (int sp = 0; sp < nsplit[bl]; ++sp)
+                for (int sp = 0; sp < (nsplit[bl] + span - 1) / span; ++sp)
                     push(MK_ATTN, 0, l, bl, g, sp, ctr(l, cl.att_in + g), att_in_tgt[g], ctr(l, cl.att_o + g * gw / o_w),
                          -1);
         // o slice sl reads the heads of the groups g with g * gw / o_w == sl
@@ -1539,9 +1557,9 @@ void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int
 // so that one pass's gate|up items fit one per CTA), the others 256-wide
 int mk_slice_atoms(int lin, int K) { return (lin == 2 && K % (MAX_ATOMS * KT) == 0) ? MAX_ATOMS : HALF_ATOMS; }
 
-size_t mk_union_bytes(int bn, int head_dim) {
+size_t mk_union_bytes(int bn, int head_dim, int att_span) {
     const size_t b = (size_t)HALF_ATOMS * bn * 128;
-    const size_t att = (size_t)2 * (head_dim / 64) * ATT_SUB_BYTES;
+    const size_t att = (size_t)att_span * 2 * (head_dim / 64) * ATT_SUB_BYTES;
     return std::max(b, att);
 }
 
@@ -1606,7 +1624,8 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
     if (P.bn > MAX_ROWS || L.pd.M > MAX_ROWS) return cudaErrorInvalidValue;
     P.tmem_cols = 32;
     while ((int)P.tmem_cols < P.bn) P.tmem_cols <<= 1;
-    const size_t uni = mk_union_bytes(P.bn, L.dm.d);
+    if (L.pd.att_span < 1 || L.pd.att_span > ATT_SPAN_MAX) return cudaErrorInvalidValue;
+    const size_t uni = mk_union_bytes(P.bn, L.dm.d, L.pd.att_span);
     const size_t static_smem = 4096;
     const long avail = (long)g_smem_optin - (long)uni - 1024 - (long)static_smem;
     // a shallow ring: what shared memory does not take stays L1 cache, which the compute warps

@@ -402,6 +402,18 @@ int draft_pass_layers(const pbd_ctx *c, int kind) {
     return (kind == PK_DRAFT && c->cfg.draft_layers > 0) ? c->cfg.draft_layers : c->cfg.n_layers;
 }
 
+// Partial results per attention split, a constant of the context (every pass of every generation
+// uses the same key partition, so verify rows stay bitwise equal to decode rows): two 64-key halves
+// on separate warps when a full-length pass's split items fit one wave of CTAs; otherwise one warp
+// per query tile over all 128 keys, which halves the partials the merge reads.
+int att_subs_of(const pbd_ctx *c) {
+    return (long)c->cfg.max_batch * c->n_splits * c->cfg.n_kv_heads > c->grid ? 1 : ATT_SUBS_MAX;
+}
+// 128-key splits per attention item: with one partial per split, an item covers two splits (one
+// query tile and split per warp, all six warps busy), halving the items of long contexts; the
+// key partition, and with it every result, is the same
+int att_span_of(const pbd_ctx *c) { return att_subs_of(c) == 1 ? ATT_SPAN_MAX : 1; }
+
 PassDesc block_pass(pbd_ctx *c, int kind) {
     PassDesc pd;
     pd.b0 = 0;
@@ -416,6 +428,7 @@ PassDesc block_pass(pbd_ctx *c, int kind) {
     pd.ro_count = kind == PK_DRAFT ? c->D : pd.R;
     pd.nl_run = draft_pass_layers(c, kind);
     pd.skip = kind == PK_DRAFT ? c->cfg.draft_skip_mask : 0;
+    pd.att_span = att_span_of(c);
     return pd;
 }
 
@@ -435,14 +448,6 @@ pbd_status upload_schedule(pbd_ctx *c, int kind, const PassDesc &pd, const std::
     CK(cudaStreamSynchronize(c->st));
     s.valid = true;
     return PBD_OK;
-}
-
-// Partial results per attention split, a constant of the context (every pass of every generation
-// uses the same key partition, so verify rows stay bitwise equal to decode rows): two 64-key halves
-// on separate warps when a full-length pass's split items fit one wave of CTAs; otherwise one warp
-// per query tile over all 128 keys, which halves the partials the merge reads.
-int att_subs_of(const pbd_ctx *c) {
-    return (long)c->cfg.max_batch * c->n_splits * c->cfg.n_kv_heads > c->grid ? 1 : ATT_SUBS_MAX;
 }
 
 MKLaunch make_launch(pbd_ctx *c, const PassDesc &pd, int kind) {
@@ -756,6 +761,7 @@ pbd_status pbd_prefill(pbd_ctx *c, int32_t batch, const int32_t *d_prompt_ids, c
             pd.b0 = b;
             pd.nb = 1;
             pd.R = rows;
+            pd.att_span = att_span_of(c);
             pd.M = rows;
             pd.adapter = 0;
             pd.mask_mode = MASK_CAUSAL;

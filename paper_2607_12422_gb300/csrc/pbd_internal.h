@@ -15,6 +15,7 @@ namespace pbd {
 constexpr int PAGE = 16;           // KV page length in tokens
 constexpr int ATT_SPLIT = 128;     // key positions per attention split (position-aligned)
 constexpr int ATT_SUBS_MAX = 2;    // partial results per split at most (its two 64-key halves)
+constexpr int ATT_SPAN_MAX = 2;    // 128-key splits per attention item at most
 constexpr int PREFILL_ROWS = 64;   // rows per prefill chunk
 constexpr int KT = 64;             // K elements per 128-byte swizzle atom row (bf16)
 constexpr int TILE_ROWS = 128;     // output features per tensor-core tile
@@ -36,6 +37,7 @@ struct PassDesc {
     int ro_count;
     int nl_run;      // decoder layers the pass runs before the final norm (the draft's early exit)
     uint64_t skip = 0;  // decoder layers below nl_run the pass skips (the draft's layer skipping)
+    int att_span = 1;   // consecutive 128-key splits one attention item covers (a context constant)
 };
 
 // Paged KV cache: [layer][page][Hkv][PAGE][d] bf16 for K and for V.
@@ -142,7 +144,7 @@ int mk_grid_size();
 void mk_counter_layout(const Dims &dm, int max_nb, CounterLayout *cl);
 void mk_build_schedule(const Dims &dm, const PassDesc &pd, const std::vector<int> &nsplit, int grid,
                        const CounterLayout &cl, std::vector<MKItem> *out, std::vector<int> *off);
-size_t mk_union_bytes(int bn, int head_dim);
+size_t mk_union_bytes(int bn, int head_dim, int att_span);
 int mk_slice_atoms(int lin, int K);  // 64-wide K atoms per work item of linear `lin`
 cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st);
 

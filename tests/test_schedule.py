@@ -279,3 +279,29 @@ def test_layer_skip_schedule():
     for bad in ((1 << S.n_layers) - 1, 1 << S.n_layers):
         with pytest.raises(pbd.PbdError):
             pbd.pbd_plan_pass(pbd.make_config(S, 16, 1, 1024, draft_skip=bad), 0, [512], 256, 152)
+
+
+@pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
+@pytest.mark.parametrize("grid", [152, 37])
+def test_attention_items_cover_the_keys(case, grid):
+    """Each (layer, sequence, KV group) has attention items 0..n-1 that together cover every
+    128-key split a pass of the generation can reach.  A context whose full-length split items
+    exceed one wave of CTAs keeps one partial result per split and lets an item cover two
+    consecutive splits (n = ceil(splits / 2)); otherwise an item is one split."""
+    _, S, D, lens, G = case
+    max_len = max(lens) + G + 8
+    cfg = pbd.make_config(S, D, len(lens), max_len)
+    items, off = pbd.pbd_plan_pass(cfg, 1, lens, G, grid)
+    op, lin, layer, a, b, c = _decode(items)
+    max_tokens = max_len + 2 * (D + 1)
+    n_splits = -(-max_tokens // 128)
+    span = 2 if len(lens) * n_splits * S.n_kv_heads > grid else 1
+    pages = -(-max_tokens // 16)
+    att = {}
+    for i in np.nonzero(op == OP_ATTN)[0]:
+        att.setdefault((int(layer[i]), int(a[i]), int(b[i])), []).append(int(c[i]))
+    assert len(att) == S.n_layers * len(lens) * S.n_kv_heads
+    for (l, bl, g), cs in att.items():
+        reach = min(lens[bl] + G + 2 * (D + 1), pages * 16)
+        splits = min(n_splits, -(-reach // 128))
+        assert sorted(cs) == list(range(-(-splits // span))), (l, bl, g, span, splits, sorted(cs))
