@@ -374,8 +374,8 @@ __device__ __noinline__ void do_embed(const MKParams &P, int m, int cw, int lane
 // two bf16 numbers rounded once to nearest even, as fp32 and then rounding gives).  A row has
 // 32 chunks of 8 elements; thread ct handles chunks ct, ct + 192, ..., so its chunk column
 // (ct % 32), and with it its gain chunk, is the same for all of them.
-__device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int slice, uint8_t *sb, float *s_rms, int ct,
-                                     int a0, bool need_rms, unsigned long long *st) {
+__device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int slice, uint8_t *sb, float *s_rms,
+                                     const uint4 *s_gain, int ct, int a0, bool need_rms, unsigned long long *st) {
     const int M = P.pd.M;
     const bool norm = lin != 1;
     const bf16 *src = norm ? P.h : P.attn;  // (the down projection's operand: build_b_act)
@@ -393,10 +393,10 @@ __device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int 
         cp_async_wait_all();
         return;
     }
-    const uint4 gv = __ldg(reinterpret_cast<const uint4 *>((lin == 0 ? P.attn_norm : P.mlp_norm) + (size_t)layer * P.dm.H + col));
     if (need_rms)  // while the copies are in flight
         for (int m = ct; m < M; m += CT) s_rms[m] = row_rms(P, m);
-    cp_async_wait_all();
+    cp_async_wait_all();  // (also the gain slice, copied before the item's inputs were ready)
+    const uint4 gv = s_gain[a0 * (KT / 8) + c];
     if (need_rms) {
         bar_compute();
         if (ct == 0) stamp_at(st, 8);
@@ -1005,6 +1005,8 @@ struct CtaState {
     // the adapter's B rows of the tile a draft's linear item reduces (tile row order: for
     // gate|up rows 0-63 gate, 64-127 up), staged at the item's start
     uint4 brows[TILE_ROWS * MAX_RANK / 8];
+    // the RMSNorm gain of the K slice a q|k|v or gate|up item stages
+    uint4 gain[MAX_ATOMS * KT / 8];
 };
 
 // ---- warp 0 lane 0: weight producer.  Walks the CTA's linear items ahead of the others and
@@ -1174,32 +1176,19 @@ __device__ __noinline__ bool item_linear(const MKParams &P, const MKItem &it, ui
                                          unsigned long long *st) {
     const int lin = it.lin, l = it.layer, t = it.a, s = it.b;
     const int na = P.katoms[lin];
-    if (DRAFT && t < P.n_main[lin] / TILE_ROWS) {
-        // the adapter's B rows of this tile: they depend only on (layer, tile), so they are copied
-        // while the operand is staged (the staging's cp.async wait covers them)
-        const int r = P.dm.r, cpr = r / 8;  // 16-byte chunks per B row
-        const bf16 *lb = P.lora_b[lin] + (size_t)l * P.lb_stride[lin];
-#pragma unroll 1
-        for (int q = ct; q < TILE_ROWS * cpr; q += CT) {
-            const int j = q / cpr, c = q % cpr;
-            const int f = lin == 2 ? (j < 64 ? t * 64 + j : P.dm.I + t * 64 + (j - 64)) : t * TILE_ROWS + j;
-            cp_async16(&S.brows[q], lb + (size_t)f * r + c * 8);
-        }
-        cp_async_commit();
-    }
     if (na <= HALF_ATOMS) {
         if (lin == 3) {
             build_b_act(P, s, uni, ct, S.tag + l, st);
             if (DRAFT) cp_async_wait_all();  // the B rows (the operand needed no copies)
         } else
-            build_b(P, lin, l, s, uni, S.rms, ct, 0, true, st);
+            build_b(P, lin, l, s, uni, S.rms, S.gain, ct, 0, true, st);
         fence_proxy_async();
         bar_compute();
         if (ct == 0) mbarrier_arrive_one(&S.b_full[0]);
     } else {
         // wide slice in two halves: when both fit, the first half's MMAs run while the second is
         // staged; else the second goes through the same area after the first half's reads
-        build_b(P, lin, l, s, uni, S.rms, ct, 0, true, st);
+        build_b(P, lin, l, s, uni, S.rms, S.gain, ct, 0, true, st);
         fence_proxy_async();
         bar_compute();
         if (ct == 0) {
@@ -1210,8 +1199,8 @@ __device__ __noinline__ bool item_linear(const MKParams &P, const MKItem &it, ui
             bar_compute();
             if (!S.ok) return false;
         }
-        build_b(P, lin, l, s, uni + (P.b_dbl ? (size_t)HALF_ATOMS * P.bn * 128 : 0), S.rms, ct, HALF_ATOMS, false,
-                nullptr);
+        build_b(P, lin, l, s, uni + (P.b_dbl ? (size_t)HALF_ATOMS * P.bn * 128 : 0), S.rms, S.gain, ct, HALF_ATOMS,
+                false, nullptr);
         fence_proxy_async();
         bar_compute();
         if (ct == 0) mbarrier_arrive_one(&S.b_full[1]);
@@ -1275,6 +1264,39 @@ __device__ __noinline__ bool item_linear(const MKParams &P, const MKItem &it, ui
     return true;
 }
 
+// ---- compute group: a linear item's constants of the layer, requested before its inputs are
+// ready (they depend on nothing computed in the pass): the RMSNorm gain of a normalised operand's
+// K slice and, in the draft, the adapter's B rows of the tile, copied to shared memory (the
+// operand staging's cp.async wait covers them); the QK-norm gains of the layer into L2.  The
+// previous item's readers of these buffers passed a barrier before this is called.
+template <bool DRAFT>
+__device__ __forceinline__ void item_consts(const MKParams &P, const MKItem &it, CtaState &S, int ct) {
+    const int lin = it.lin, l = it.layer, t = it.a;
+    bool any = false;
+    if (DRAFT && t < P.n_main[lin] / TILE_ROWS) {
+        const int r = P.dm.r, cpr = r / 8;  // 16-byte chunks per B row
+        const bf16 *lb = P.lora_b[lin] + (size_t)l * P.lb_stride[lin];
+#pragma unroll 1
+        for (int q = ct; q < TILE_ROWS * cpr; q += CT) {
+            const int j = q / cpr, c = q % cpr;
+            const int f = lin == 2 ? (j < 64 ? t * 64 + j : P.dm.I + t * 64 + (j - 64)) : t * TILE_ROWS + j;
+            cp_async16(&S.brows[q], lb + (size_t)f * r + c * 8);
+        }
+        any = true;
+    }
+    if (lin == 0 || lin == 2) {
+        const int n = P.katoms[lin] * (KT / 8);  // 16-byte chunks of the slice's gain
+        const bf16 *g = (lin == 0 ? P.attn_norm : P.mlp_norm) + (size_t)l * P.dm.H + (size_t)it.b * n * 8;
+        if (ct < n) cp_async16(&S.gain[ct], g + ct * 8);
+        any = true;
+    }
+    if (lin == 0 && ct < 2 * P.dm.d / 64) {  // the q and k gains: 128-byte lines
+        const int kind = ct / (P.dm.d / 64), line = ct % (P.dm.d / 64);
+        prefetch_l2((kind ? P.k_norm : P.q_norm) + (size_t)l * P.dm.d + line * 64);
+    }
+    if (any) cp_async_commit();
+}
+
 // ---- compute group (warps 2-7): dependency waits, operand staging, epilogues, reductions,
 // attention; the attention's cached pages are requested by warp CT_PAGES / 32 while thread 0 polls
 // the item's inputs
@@ -1302,6 +1324,7 @@ __device__ __noinline__ void run_compute(const MKParams &P, const MKItem *my, in
             attn_pages(P, it.layer, it.a, it.b, it.c, 0, uni, &S.att_bar, lane);
             att_pend = true;
         }
+        if (it.op == MK_LINEAR) item_consts<DRAFT>(P, it, S, ct);
         if (ct == 0) S.flag = wait_deps(P, it) ? 1 : 0;
         bar_compute();
         if (!S.flag) break;
@@ -1321,6 +1344,7 @@ __device__ __noinline__ void run_compute(const MKParams &P, const MKItem *my, in
         }
         if (!ok) break;
     }
+    cp_async_wait_all();  // an item left on abort may have requested its constants
     if (tr && ct == 0 && n_my > 0) tr[MK_STAMPS * (n_my - 1) + 3] = globaltimer_ns();
     if (ct == CT_PAGES && att_pend) {
         // the pass ended before the split waited for its pages: complete the phase's arrival and
@@ -1626,7 +1650,7 @@ cudaError_t launch_pass_kernel(const MKLaunch &L, cudaStream_t st) {
     while ((int)P.tmem_cols < P.bn) P.tmem_cols <<= 1;
     if (L.pd.att_span < 1 || L.pd.att_span > ATT_SPAN_MAX) return cudaErrorInvalidValue;
     const size_t uni = mk_union_bytes(P.bn, L.dm.d, L.pd.att_span);
-    const size_t static_smem = 4096;
+    const size_t static_smem = sizeof(CtaState) + 1024;
     const long avail = (long)g_smem_optin - (long)uni - 1024 - (long)static_smem;
     // a shallow ring: what shared memory does not take stays L1 cache, which the compute warps
     // stack frames, spills and read-only loads need more than the weight stream needs depth
