@@ -1223,6 +1223,17 @@ __device__ __noinline__ bool item_linear(const MKParams &P, const MKItem &it, ui
             const int n_total = P.n_main[lin] + P.lora_rows[lin];
             unsigned long long *d = P.part[lin] + (size_t)s * P.part_rows * n_total + t * TILE_ROWS + row;
             const uint32_t taddr = tmem + ((uint32_t)(quarter * 32) << 16);
+            if (P.pd.M <= 32) {  // one load of all token columns
+                uint32_t v[32];
+                tmem_ld_32cols(taddr, v);
+                tmem_ld_wait();
+                const int nc = mine ? P.pd.M : 0;
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                    if (j < nc) st_tagged(d, v[j], tag);
+                    d += n_total;
+                }
+            } else
 #pragma unroll 1
             for (int c0 = 0; c0 < P.pd.M; c0 += 8) {
                 uint32_t v[8];
