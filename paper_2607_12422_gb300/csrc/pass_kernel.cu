@@ -395,7 +395,7 @@ __device__ __noinline__ void build_b(const MKParams &P, int lin, int layer, int 
     }
     if (need_rms)  // while the copies are in flight
         for (int m = ct; m < M; m += CT) s_rms[m] = row_rms(P, m);
-    cp_async_wait_all();  // (also the gain slice, copied before the item's inputs were ready)
+    cp_async_wait_all();
     const uint4 gv = s_gain[a0 * (KT / 8) + c];
     if (need_rms) {
         bar_compute();
@@ -1277,9 +1277,10 @@ __device__ __noinline__ bool item_linear(const MKParams &P, const MKItem &it, ui
 
 // ---- compute group: a linear item's constants of the layer, requested before its inputs are
 // ready (they depend on nothing computed in the pass): the RMSNorm gain of a normalised operand's
-// K slice and, in the draft, the adapter's B rows of the tile, copied to shared memory (the
-// operand staging's cp.async wait covers them); the QK-norm gains of the layer into L2.  The
-// previous item's readers of these buffers passed a barrier before this is called.
+// K slice and, in the draft, the adapter's B rows of the tile, copied to shared memory (each thread
+// waits for its own copies before the barrier that follows the input wait, which publishes them to
+// the threads that read them); the QK-norm gains of the layer into L2.  The previous item's
+// readers of these buffers passed a barrier before this is called.
 template <bool DRAFT>
 __device__ __forceinline__ void item_consts(const MKParams &P, const MKItem &it, CtaState &S, int ct) {
     const int lin = it.lin, l = it.layer, t = it.a;
@@ -1337,6 +1338,7 @@ __device__ __noinline__ void run_compute(const MKParams &P, const MKItem *my, in
         }
         if (it.op == MK_LINEAR) item_consts<DRAFT>(P, it, S, ct);
         if (ct == 0) S.flag = wait_deps(P, it) ? 1 : 0;
+        cp_async_wait_all();  // the constants each thread requested, published by the barrier
         bar_compute();
         if (!S.flag) break;
         if (ct == 0 && st) st[1] = st[2] = globaltimer_ns();
