@@ -586,7 +586,7 @@ __device__ __noinline__ void reduce_residual(const MKParams &P, int lin, int lay
         uint2 *hp = reinterpret_cast<uint2 *>(P.h + (size_t)m * H + f0);
         const uint2 hraw = __ldcg(hp);
         float acc[5];
-        sum_parts<2, AD, AD ? 4 : 8>(P, lin, m, f0, P.n_main[lin] + (lane < r ? lane : 0), acc, tag);
+        sum_parts<2, AD, AD ? 4 : 12>(P, lin, m, f0, P.n_main[lin] + (lane < r ? lane : 0), acc, tag);
         unsigned long long *sw = (cw == 0 && m == m0 && lane == 0) ? st : nullptr;  // first row's sub-steps
         stamp_at(sw, 9);
         float u[MAX_RANK];
