@@ -717,7 +717,7 @@ __device__ __noinline__ void attn_pages(const MKParams &P, int layer, int bl, in
 // split has two partial results; every unit is a partial result (m, l, O) that the merge combines
 // in key order; the partition of the keys does not depend on the span.  Within a unit the keys go
 // in chunks of 32 with a running maximum (online softmax): scores by bf16 mma.sync, the row maximum
-// and the weights in fp32, P (weights) in fp16 against V converted to fp16, O in fp32.  The loop
+// and the weights in fp32, P (weights) rounded to bf16 against the cached bf16 V, O in fp32.  The loop
 // over chunks is not unrolled: the code stays small enough for the instruction cache.
 template <int DH, bool BLK>
 __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, int g, int s, uint8_t *smem,
@@ -738,27 +738,20 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
     const int n_mt = (QV + 15) / 16;
     const bool landed = mbar_wait_mk(bar, parity, P, DEV_TIMEOUT_LOAD);
     if (stamp && ct == 0) stamp[4] = globaltimer_ns();
-    // V to fp16 in place (each 16-byte chunk independently; the swizzle layout is unchanged).
-    // Rows of keys at or past T become zeros: their weights are 0, but their slots hold whatever
-    // the cache held (a page's tail beyond the sequence, or pages not loaded at all), and 0 times
-    // an Inf or NaN there would poison the sum.  Their K rows are masked out of the scores.
-    constexpr int VCH = SUBS * ATT_SUB_BYTES / 16;  // 16-byte chunks of one split's V
+    // V rows of keys at or past T that a 32-key chunk reads (the rest of the last chunk) become
+    // zeros: their weights are 0, but their slots hold whatever the cache held (a page's tail
+    // beyond the sequence, or pages not loaded at all), and 0 times an Inf or NaN there would
+    // poison the sum.  Their K rows are masked out of the scores.  Only the split that holds T
+    // has such rows: keys T - k0 up to the next multiple of 32, all head-dimension halves.
+    {
+        const int kz0 = T - (sp0 + nsx - 1) * ATT_SPLIT;  // in the item's last split holding keys
+        const int kz1 = min(ATT_SPLIT, (kz0 + 31) & ~31);
+        uint8_t *sVl = smem + (nsx - 1) * SPB + SUBS * ATT_SUB_BYTES;
 #pragma unroll 1
-    for (int idx = ct; idx < nsx * VCH; idx += CT) {
-        const int sp = idx / VCH, w = idx % VCH;
-        uint4 *p4 = reinterpret_cast<uint4 *>(smem + sp * SPB + SUBS * ATT_SUB_BYTES + w * 16);
-        const int key = (w % (ATT_SUB_BYTES / 16)) >> 3;  // 8 chunks of 16 bytes per key row
-        uint4 v4 = make_uint4(0, 0, 0, 0);
-        if ((sp0 + sp) * ATT_SPLIT + key < T) {
-            v4 = *p4;
-            uint32_t *w = reinterpret_cast<uint32_t *>(&v4);
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[e]));
-                w[e] = pack_half2(f.x, f.y);
-            }
+        for (int idx = ct; idx < (kz1 - kz0) * SUBS * 8; idx += CT) {
+            const int row = kz0 + idx / (SUBS * 8), c = idx % (SUBS * 8);
+            *reinterpret_cast<uint4 *>(sVl + (c >> 3) * ATT_SUB_BYTES + row * 128 + (c & 7) * 16) = make_uint4(0, 0, 0, 0);
         }
-        *p4 = v4;
     }
     bar_compute();
     if (stamp && ct == 0) stamp[5] = globaltimer_ns();
@@ -864,10 +857,10 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
 #pragma unroll
             for (int kstep = 0; kstep < CN / 2; ++kstep) {
                 uint32_t pa[4];
-                pa[0] = pack_half2(sc[2 * kstep][0], sc[2 * kstep][1]);
-                pa[1] = pack_half2(sc[2 * kstep][2], sc[2 * kstep][3]);
-                pa[2] = pack_half2(sc[2 * kstep + 1][0], sc[2 * kstep + 1][1]);
-                pa[3] = pack_half2(sc[2 * kstep + 1][2], sc[2 * kstep + 1][3]);
+                pa[0] = pack_bf162(sc[2 * kstep][0], sc[2 * kstep][1]);
+                pa[1] = pack_bf162(sc[2 * kstep][2], sc[2 * kstep][3]);
+                pa[2] = pack_bf162(sc[2 * kstep + 1][0], sc[2 * kstep + 1][1]);
+                pa[3] = pack_bf162(sc[2 * kstep + 1][2], sc[2 * kstep + 1][3]);
                 const int vrow = kb + c0 + kstep * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
 #pragma unroll
                 for (int dt = 0; dt < DT; dt += 2) {
@@ -877,8 +870,8 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
                     asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
                                  : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
                                  : "r"(addr));
-                    mma_m16n8k16_f16(oc[dt], pa, r0, r1);
-                    mma_m16n8k16_f16(oc[dt + 1], pa, r2, r3);
+                    mma_m16n8k16_bf16(oc[dt], pa, r0, r1);
+                    mma_m16n8k16_bf16(oc[dt + 1], pa, r2, r3);
                 }
             }
         }
