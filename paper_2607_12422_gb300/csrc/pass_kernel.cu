@@ -738,22 +738,6 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
     const int n_mt = (QV + 15) / 16;
     const bool landed = mbar_wait_mk(bar, parity, P, DEV_TIMEOUT_LOAD);
     if (stamp && ct == 0) stamp[4] = globaltimer_ns();
-    // V rows of keys at or past T that a 32-key chunk reads (the rest of the last chunk) become
-    // zeros: their weights are 0, but their slots hold whatever the cache held (a page's tail
-    // beyond the sequence, or pages not loaded at all), and 0 times an Inf or NaN there would
-    // poison the sum.  Their K rows are masked out of the scores.  Only the split that holds T
-    // has such rows: keys T - k0 up to the next multiple of 32, all head-dimension halves.
-    {
-        const int kz0 = T - (sp0 + nsx - 1) * ATT_SPLIT;  // in the item's last split holding keys
-        const int kz1 = min(ATT_SPLIT, (kz0 + 31) & ~31);
-        uint8_t *sVl = smem + (nsx - 1) * SPB + SUBS * ATT_SUB_BYTES;
-#pragma unroll 1
-        for (int idx = ct; idx < (kz1 - kz0) * SUBS * 8; idx += CT) {
-            const int row = kz0 + idx / (SUBS * 8), c = idx % (SUBS * 8);
-            *reinterpret_cast<uint4 *>(sVl + (c >> 3) * ATT_SUB_BYTES + row * 128 + (c & 7) * 16) = make_uint4(0, 0, 0, 0);
-        }
-    }
-    bar_compute();
     if (stamp && ct == 0) stamp[5] = globaltimer_ns();
     if (!landed) return;
     const int gq = lane >> 2, tq = lane & 3;
@@ -862,6 +846,18 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
                 pa[2] = pack_bf162(sc[2 * kstep + 1][0], sc[2 * kstep + 1][1]);
                 pa[3] = pack_bf162(sc[2 * kstep + 1][2], sc[2 * kstep + 1][3]);
                 const int vrow = kb + c0 + kstep * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+                // V of keys at or past T is set to zero in the fragments: their weights are 0, but
+                // their rows hold whatever the cache or shared memory held (a page's tail beyond the
+                // sequence, or pages not loaded at all), and 0 times an Inf or NaN there would
+                // poison the sum.  Fragment registers b0 / b1 hold keys 2 tq, 2 tq + 1 / + 8, + 9 of
+                // the 16-key step, the lower key in the low half.
+                const int kst = k0 + kb + c0 + kstep * 16;  // first key of the step
+                uint32_t ma = 0xFFFFFFFFu, mb = 0xFFFFFFFFu;
+                if (kst + 16 > T) {  // warp-uniform: only the steps that reach T
+                    const int ka = kst + 2 * tq;
+                    ma = (ka < T ? 0x0000FFFFu : 0u) | (ka + 1 < T ? 0xFFFF0000u : 0u);
+                    mb = (ka + 8 < T ? 0x0000FFFFu : 0u) | (ka + 9 < T ? 0xFFFF0000u : 0u);
+                }
 #pragma unroll
                 for (int dt = 0; dt < DT; dt += 2) {
                     const int vcol = dt * 8 + (lane >> 4) * 8;
@@ -870,8 +866,8 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
                     asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
                                  : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
                                  : "r"(addr));
-                    mma_m16n8k16_bf16(oc[dt], pa, r0, r1);
-                    mma_m16n8k16_bf16(oc[dt + 1], pa, r2, r3);
+                    mma_m16n8k16_bf16(oc[dt], pa, r0 & ma, r1 & mb);
+                    mma_m16n8k16_bf16(oc[dt + 1], pa, r2 & ma, r3 & mb);
                 }
             }
         }
