@@ -148,6 +148,16 @@ def gen_base_weights(shape: ModelShape, seed: int = SEED_WEIGHTS) -> Dict[str, n
     return w
 
 
+def with_random_norm_gains(w: Dict[str, np.ndarray], seed: int = SEED_WEIGHTS + 7) -> Dict[str, np.ndarray]:
+    """A copy of base weights whose RMSNorm gains (final, attn, mlp, q, k) are drawn uniformly from
+    [0.5, 1.5) and rounded to bf16, in that order from one PCG64 stream; the rest is shared."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    out = dict(w)
+    for k in ("final_norm", "attn_norm", "mlp_norm", "q_norm", "k_norm"):
+        out[k] = bf16_bits(rng.uniform(0.5, 1.5, size=w[k].shape).astype(np.float32))
+    return out
+
+
 def gen_adapter(shape: ModelShape, seed: int = SEED_ADAPTER, zero_B: bool = False) -> Dict[str, np.ndarray]:
     """Adapter weights: per linear A [nl, r, in] and B [nl, out, r], plus mask_embed [H].
 

@@ -39,6 +39,26 @@ def _check_ids(ids, ref_logits, tol=TOL):
             assert ref_logits[j][best] - ref_logits[j][t] <= tol, (j, t, best)
 
 
+def test_lockstep_rounds_random_norm_gains(env):
+    """Six lockstep rounds with every RMSNorm gain drawn from [0.5, 1.5) (the default synthetic
+    gains are all 1, which would hide a gain applied to the wrong column or not at all): logits
+    within 3e-2, every verify id equal to the oracle's argmax."""
+    S, pbd = env["S"], env["pbd"]
+    base = synth.with_random_norm_gains(env["base"])
+    assert not np.all(base["attn_norm"] == env["base"]["attn_norm"])
+    m = oracle.OracleModel(S, base, env["ad"])
+    eng = pbd.Engine(S, base, env["ad"], block_D=D, max_batch=1, max_seq_len=256)
+    prompt = env["prompts"][0]
+    seqs = {0: _parity.Seq(m, None, prompt, D, 6)}
+    _parity.start(eng, [prompt], seqs, 64, "tiny-b1-d16-p64-g64-random-gains")
+    n0 = len(_parity.RECORDS)
+    _parity.rounds(eng, seqs, 6, "tiny-b1-d16-p64-g64-random-gains")
+    eng.close()
+    new = _parity.RECORDS[n0:]
+    assert all(r["bound"] == TOL for r in new)
+    assert sum(r["id_mismatches"] for r in new if r["pass_kind"] == "verify") == 0
+
+
 def test_round_matches_oracle(env):
     eng, m, prompt = env["eng"], env["model"], env["prompts"][0]
     P = len(prompt)

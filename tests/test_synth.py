@@ -53,3 +53,16 @@ def test_workloads_shapes():
     p = synth.gen_prompts(w.shape, w.prompt_lens)
     assert [len(x) for x in p] == list(w.prompt_lens)
     assert all(x.min() >= 0 and x.max() < w.shape.vocab for x in p)
+
+
+def test_random_norm_gains():
+    a = synth.gen_base_weights(synth.TINY)
+    r = synth.with_random_norm_gains(a)
+    r2 = synth.with_random_norm_gains(a)
+    for k in ("final_norm", "attn_norm", "mlp_norm", "q_norm", "k_norm"):
+        g = synth.bf16_to_f32(r[k])
+        assert r[k].shape == a[k].shape and np.array_equal(r[k], r2[k])
+        assert g.min() >= 0.5 and g.max() <= 1.5 and len(np.unique(g)) > 10
+    for k in synth.LINEARS:
+        assert r["w" + k] is a["w" + k]
+    assert np.all(a["attn_norm"] == 0x3F80)  # the input dict is not modified
