@@ -74,6 +74,11 @@ typedef struct {
                                  writes no K/V there); 0 = none.  Bits at or above n_layers must be
                                  clear, and the draft must keep at least one layer (together with
                                  draft_layers) */
+    int32_t max_ctas;         /* CTAs of the persistent pass kernel: 0 = one per SM; otherwise at most
+                                 max_ctas (leaving SMs to other work).  It must be at least the largest
+                                 number of K slices of one linear, whose reductions wait for one
+                                 another and so must sit on distinct CTAs: pbd_create fails with
+                                 PBD_ERR_INVALID_ARG below that */
 } pbd_config;
 
 /* Backbone weights: bf16, row-major [out, in] per linear, stacked over layers.  They are

@@ -181,6 +181,7 @@ bool valid_config(const pbd_config *cfg, std::string *why) {
     if (k.draft_unanchored != 0 && k.draft_unanchored != 1) return bad("draft_unanchored must be 0 or 1");
     if (k.n_layers < 64 && (k.draft_skip_mask >> k.n_layers) != 0)
         return bad("draft_skip_mask has bits at or above n_layers");
+    if (k.max_ctas < 0 || k.max_ctas > 256) return bad("max_ctas must be in [0, 256]");
     {
         const int E = k.draft_layers > 0 ? k.draft_layers : k.n_layers;
         int kept = 0;
@@ -684,6 +685,18 @@ pbd_status pbd_create(const pbd_config *cfg, const pbd_base_weights *base, const
     if (c->grid <= 0 || c->grid > 256) {
         delete c;
         return fail(nullptr, PBD_ERR_CUDA, "cannot query the SM count");
+    }
+    if (cfg->max_ctas > 0) c->grid = std::min(c->grid, cfg->max_ctas);
+    {
+        // the K slices of one tile reduce each other's partial sums: one CTA each
+        int need = 1;
+        for (int lin = 0; lin < 4; ++lin)
+            need = std::max(need, lin_K(*cfg, lin) / (mk_slice_atoms(lin, lin_K(*cfg, lin)) * KT));
+        if (c->grid < need) {
+            const int g = c->grid;
+            delete c;
+            return fail(nullptr, PBD_ERR_INVALID_ARG, "max_ctas %d below the %d K slices of one linear", g, need);
+        }
     }
     uint8_t *wb = static_cast<uint8_t *>(d_workspace);
     uint8_t *b1024 = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(wb) + ALIGN - 1) & ~(uintptr_t)(ALIGN - 1));

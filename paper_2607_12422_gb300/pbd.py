@@ -37,7 +37,7 @@ class pbd_config(C.Structure):
                 ("lora_rank", C.c_int32), ("lora_scale", C.c_float), ("block_D", C.c_int32),
                 ("max_batch", C.c_int32), ("max_seq_len", C.c_int32), ("page_size", C.c_int32),
                 ("draft_layers", C.c_int32), ("denoise_steps", C.c_int32), ("draft_unanchored", C.c_int32),
-                ("draft_skip_mask", C.c_uint64)]
+                ("draft_skip_mask", C.c_uint64), ("max_ctas", C.c_int32)]
 
 
 class pbd_base_weights(C.Structure):
@@ -216,12 +216,12 @@ def pbd_op_lm_head_argmax(x, E, want_logits: bool = False):
 
 
 def make_config(shape, block_D: int, max_batch: int, max_seq_len: int, draft_layers: int = 0,
-                denoise_steps: int = 1, anchored: bool = True, draft_skip: int = 0) -> pbd_config:
+                denoise_steps: int = 1, anchored: bool = True, draft_skip: int = 0, max_ctas: int = 0) -> pbd_config:
     """pbd_config for a model shape; the draft variant defaults to the method of Section 3."""
     return pbd_config(shape.n_layers, shape.hidden, shape.n_q_heads, shape.n_kv_heads, shape.head_dim,
                       shape.intermediate, shape.vocab, shape.rms_eps, shape.rope_theta, shape.lora_rank,
                       shape.lora_alpha / shape.lora_rank, block_D, max_batch, max_seq_len, 16,
-                      draft_layers, denoise_steps, 0 if anchored else 1, draft_skip)
+                      draft_layers, denoise_steps, 0 if anchored else 1, draft_skip, max_ctas)
 
 
 def pbd_plan_pass(cfg: pbd_config, kind: int, prompt_lens: Sequence[int], max_new: int, grid: int,
@@ -249,7 +249,8 @@ class Engine:
 
     def __init__(self, shape, base: Dict[str, np.ndarray], adapter: Dict[str, np.ndarray], block_D: int,
                  max_batch: int, max_seq_len: int, device: str = "cuda:0", keep_host_weights: bool = False,
-                 draft_layers: int = 0, denoise_steps: int = 1, anchored: bool = True, draft_skip: int = 0):
+                 draft_layers: int = 0, denoise_steps: int = 1, anchored: bool = True, draft_skip: int = 0,
+                 max_ctas: int = 0):
         import torch
         self.torch = torch
         self.lib = load()
@@ -257,7 +258,7 @@ class Engine:
         self.D = block_D
         self.device = torch.device(device)
         self.cfg = make_config(shape, block_D, max_batch, max_seq_len, draft_layers, denoise_steps, anchored,
-                               draft_skip)
+                               draft_skip, max_ctas)
         need = self.lib.pbd_workspace_bytes(C.byref(self.cfg))
         if need == 0:
             raise PbdError(1, "configuration rejected by pbd_workspace_bytes")

@@ -59,6 +59,27 @@ def test_lockstep_rounds_random_norm_gains(env):
     assert sum(r["id_mismatches"] for r in new if r["pass_kind"] == "verify") == 0
 
 
+def test_few_ctas_last_item_merges_lockstep(env):
+    """The pass kernel on 4 CTAs (many items per CTA) with a 1000-token prompt: each (sequence, KV
+    head) then has more attention items than CTAs, so the last item to finish merges all of them
+    (the path long batched contexts take on the full GPU).  Three lockstep rounds at 3e-2."""
+    S, pbd = env["S"], env["pbd"]
+    P, G = 1000, 48
+    cfg = pbd.make_config(S, D, 1, P + G + 8, max_ctas=4)
+    items, _ = pbd.pbd_plan_pass(cfg, 1, [P], G, 4)
+    op, c, b = items[:, 0] & 0xFF, items[:, 3], items[:, 2]
+    layer0 = (items[:, 0] >> 16) == 0
+    assert min(int(c[(op == 2) & layer0 & (b == g)].max()) + 1 for g in range(S.n_kv_heads)) > 4
+    prompt = synth.gen_prompts(S, [P], seed=11)[0]
+    eng = pbd.Engine(S, env["base"], env["ad"], block_D=D, max_batch=1, max_seq_len=P + G + 8, max_ctas=4)
+    seqs = {0: _parity.Seq(env["model"], None, prompt, D, 3)}
+    _parity.start(eng, [prompt], seqs, G, "tiny-b1-d16-p1000-4ctas")
+    n0 = len(_parity.RECORDS)
+    _parity.rounds(eng, seqs, 3, "tiny-b1-d16-p1000-4ctas")
+    eng.close()
+    assert all(r["bound"] == TOL for r in _parity.RECORDS[n0:])
+
+
 def test_round_matches_oracle(env):
     eng, m, prompt = env["eng"], env["model"], env["prompts"][0]
     P = len(prompt)

@@ -45,8 +45,11 @@ def test_workspace_size_and_config_validation(lib):
     # draft variants: early exit within the depth, at most 8 denoising steps, a 0/1 readout flag
     var = pbd.make_config(synth.TINY, 16, 4, 256, draft_layers=1, denoise_steps=2, anchored=False)
     assert lib.pbd_workspace_bytes(C.byref(var)) == lib.pbd_workspace_bytes(C.byref(tiny))
+    # a CTA limit does not change the workspace (sized for 256 CTAs)
+    capped = pbd.make_config(synth.TINY, 16, 4, 256, max_ctas=8)
+    assert lib.pbd_workspace_bytes(C.byref(capped)) == lib.pbd_workspace_bytes(C.byref(tiny))
     for field, value in (("draft_layers", synth.TINY.n_layers + 1), ("draft_layers", -1), ("denoise_steps", 9),
-                         ("draft_unanchored", 2)):
+                         ("draft_unanchored", 2), ("max_ctas", -1), ("max_ctas", 257)):
         bad = pbd.make_config(synth.TINY, 16, 4, 256)
         setattr(bad, field, value)
         assert lib.pbd_workspace_bytes(C.byref(bad)) == 0, field

@@ -305,3 +305,15 @@ def test_attention_items_cover_the_keys(case, grid):
         reach = min(lens[bl] + G + 2 * (D + 1), pages * 16)
         splits = min(n_splits, -(-reach // 128))
         assert sorted(cs) == list(range(-(-splits // span))), (l, bl, g, span, splits, sorted(cs))
+
+
+@pytest.mark.parametrize("kind", [0, 1, 2])
+def test_schedule_on_few_ctas(kind):
+    """Four CTAs (the fewest the tiny model allows: its down projection has three K slices) and a
+    1000-token prompt: many items per CTA, and more attention items per head group than CTAs (the
+    last item merges them all, so they need not sit on distinct CTAs)."""
+    S, grid, lens, G = synth.TINY, 4, [1000], 48
+    cfg = pbd.make_config(S, 16, 1, lens[0] + G + 8, max_ctas=grid)
+    items, off = pbd.pbd_plan_pass(cfg, kind, lens, G, grid)
+    _check(S, items, off, grid, S.n_layers, [256, 256, 256, 256])
+    _check_counters(items, off, grid)
