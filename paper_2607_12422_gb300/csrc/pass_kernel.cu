@@ -837,7 +837,7 @@ __device__ __noinline__ void attn_split(const MKParams &P, int layer, int bl, in
                     l0 += sc[nt][e];
                     l1 += sc[nt][2 + e];
                 }
-            // P as the fp16 A fragments of two 16-key steps
+            // P as the bf16 A fragments of two 16-key steps
 #pragma unroll
             for (int kstep = 0; kstep < CN / 2; ++kstep) {
                 uint32_t pa[4];

@@ -39,7 +39,8 @@ def summarize(items, tr):
                                "work_us_med": float(np.median(work)), "post_us_med": float(np.median(post)),
                                "item_us_max": float((t[sel, 3] - t[sel, 0]).max())}
         # sub-stamps 4..7 (0 = not reached): linear = operand staged, accumulator ready, partials
-        # stored, reduced; attention = K/V landed, V converted, all splits stored, merged
+        # stored, reduced; attention = K/V landed, pages ready for the compute (the same instant
+        # now that V needs no conversion), all splits stored, merged
         sub = {}
         labels = (("staged", "acc_ready", "counted", "reduced") if name not in ("attn",)
                   else ("landed", "converted", "counted", "merged"))
