@@ -243,11 +243,17 @@ __device__ __forceinline__ float row_rms(const MKParams &P, int m) {
 struct BRow {
     uint4 w[MAX_RANK / 8];
 };
-// the B row of local tile row j, from the tile's B rows staged in shared memory (r / 8 chunks each)
+// The tile's B rows in shared memory: row j's r / 8 chunks of 16 bytes start at chunk
+// j * (r / 8) + j / 4, i.e. 16 bytes of padding after every 4 rows.  Lane l reads rows 4l + e (or
+// 2l + e), so without the padding the 8 lanes of a 128-byte load phase would hit the same four
+// banks (8-way conflicts, with all six warps contending for the SM's shared-memory pipe: ~1700
+// cycles for the four rows' dot products, ~750 padded).
+__device__ __forceinline__ int brow_chunk(int j, int r) { return j * (r / 8) + (j >> 2); }
+// the B row of local tile row j, from the tile's B rows staged in shared memory
 __device__ __forceinline__ BRow smem_brow(const uint4 *brows, int j, int r) {
     BRow b;
 #pragma unroll
-    for (int q = 0; q < MAX_RANK / 8; ++q) b.w[q] = q * 8 < r ? brows[j * (r / 8) + q] : make_uint4(0, 0, 0, 0);
+    for (int q = 0; q < MAX_RANK / 8; ++q) b.w[q] = q * 8 < r ? brows[brow_chunk(j, r) + q] : make_uint4(0, 0, 0, 0);
     return b;
 }
 __device__ __forceinline__ float lora_dot_w(const float (&u)[MAX_RANK], const BRow &b, int r) {
@@ -993,7 +999,7 @@ struct CtaState {
     int rowpos[MAX_ROWS], rowkv[MAX_ROWS];
     // the adapter's B rows of the tile a draft's linear item reduces (tile row order: for
     // gate|up rows 0-63 gate, 64-127 up), staged at the item's start
-    uint4 brows[TILE_ROWS * MAX_RANK / 8];
+    uint4 brows[TILE_ROWS * MAX_RANK / 8 + TILE_ROWS / 4];
     // the RMSNorm gain of the K slice a q|k|v or gate|up item stages
     uint4 gain[MAX_ATOMS * KT / 8];
 };
@@ -1281,7 +1287,7 @@ __device__ __forceinline__ void item_consts(const MKParams &P, const MKItem &it,
         for (int q = ct; q < TILE_ROWS * cpr; q += CT) {
             const int j = q / cpr, c = q % cpr;
             const int f = lin == 2 ? (j < 64 ? t * 64 + j : P.dm.I + t * 64 + (j - 64)) : t * TILE_ROWS + j;
-            cp_async16(&S.brows[q], lb + (size_t)f * r + c * 8);
+            cp_async16(&S.brows[brow_chunk(j, r) + c], lb + (size_t)f * r + c * 8);
         }
         any = true;
     }
