@@ -14,9 +14,9 @@
 //               depend on nothing, so the ring fills across phase boundaries.
 //   warp 1      MMA issuer: per linear item, 4 x 4 tcgen05.mma (128 x BN x 16, bf16 -> fp32) into
 //               a TMEM accumulator; frees ring slots with tcgen05.commit.
-//   warps 2-7   compute group: dependency waits, operand staging (RMSNorm applied on the fly
-//               while building the activation tile in the swizzle layout), the TMEM epilogue
-//               (warps 4-7, one per TMEM lane quarter), attention, split reductions.
+//   warps 2-7   compute group: dependency waits, operand staging (RMSNorm applied in place in
+//               the activation tile's swizzle layout), the TMEM epilogue (warps 4-7, one per TMEM
+//               lane quarter), attention, split reductions.
 //
 // A linear is split along K into 256-wide slices (512 for gate|up; fixed per linear, independent
 // of the row count).  Each slice item stores its fp32 partial sums as 64-bit words tagged with
@@ -31,10 +31,11 @@
 // themselves.  Each reduction then counts once, with release semantics, on the counter its
 // consumers poll (attention inputs per KV head, the residual), except gate|up: SiLU(gate) * up
 // goes out as tagged words that the down projection's operand staging polls.
-// Attention items cover (sequence, KV head, 128-key split); when the splits sit on distinct
-// CTAs they wait for one another and each merges a share of the rows, else the last one
-// merges all.  RMSNorm statistics are summed per 128-feature
-// tile in one fixed order, so every row's arithmetic is independent of the pass it is in.
+// Attention items cover (sequence, KV head, att_span consecutive 128-key splits: one, or two in
+// long contexts); when a group's items sit on distinct CTAs they wait for one another and each
+// merges a share of the rows, else the last one merges all.  RMSNorm statistics are summed per
+// 128-feature tile in one fixed order, so every row's arithmetic is independent of the pass it
+// is in.
 #include <algorithm>
 #include <cmath>
 #include <vector>

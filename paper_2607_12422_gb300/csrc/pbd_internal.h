@@ -81,8 +81,9 @@ enum MKOp : uint8_t { MK_EMBED = 0, MK_LINEAR = 1, MK_ATTN = 2, MK_FINAL = 3 };
 constexpr int MK_STAMPS = 16;
 
 // One work item of a pass.  MK_LINEAR: lin (0 q|k|v, 1 o, 2 gate|up, 3 down), a = row tile
-// (the adapter tile is the last one), b = 256-wide K slice.  MK_ATTN: a = sequence in the pass,
-// b = KV head, c = 128-key split.  MK_EMBED: a = row.  MK_FINAL: a = read-out index, b = row.
+// (the adapter tile is the last one), b = K slice.  MK_ATTN: a = sequence in the pass, b = KV
+// head, c = item index (splits c * att_span .. c * att_span + att_span - 1 of 128 keys each).
+// MK_EMBED: a = row.  MK_FINAL: a = read-out index, b = row.
 // Dependencies, worked out on the host: the item waits until counter wait_off (an index into the
 // pass's counters, -1: none) reaches wait_tgt, and once its result is stored it adds one to each
 // counter rel[k] >= 0 (a reduction, an embedded row, an attention merge).
